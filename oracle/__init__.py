@@ -1,0 +1,133 @@
+"""fp64 CPU oracle for the selective-scan layer core (test infrastructure).
+
+Only the test suite, ``__graft_entry__.smoke()`` and the benchmark's CPU
+baseline leg may import this package. It shares no code with the CUDA library
+and never imports it. The arithmetic lives in ``mb_oracle.c`` (plain C, fp64,
+sequential in time); this module compiles it with gcc and marshals numpy
+arrays to it.
+
+Functions (MambaByte, Eq. 2-3, discretisation appendix, Table 6, Algorithm 1):
+
+* ``scan``     - the layer core over a whole span: y, final state, and
+                 optionally every per-position state (verify).
+* ``step``     - one recurrent decode step (a scan of length 1).
+* ``rollback`` - keep the state after ``accept`` drafted bytes.
+
+Inputs are widened exactly to float64 before the call (bf16 and fp32 values
+are exactly representable in fp64).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "mb_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libmb_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+B_EULER, B_ZOH = 0, 1
+
+
+def build(force: bool = False) -> str:
+    """Compile mb_oracle.c into _build/libmb_oracle.so (gcc, OpenMP)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    subprocess.run(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp",
+                    "-fno-fast-math", "-ffp-contract=off", _SRC, "-o", tmp, "-lm"],
+                   check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            dp = ctypes.POINTER(ctypes.c_double)
+            i64 = ctypes.c_int64
+            lib.oracle_scan.argtypes = [i64, i64, i64, i64] + [dp] * 9 + [ctypes.c_int, dp, dp, dp,
+                                                                         ctypes.c_int]
+            lib.oracle_scan.restype = ctypes.c_int
+            lib.oracle_rollback.argtypes = [i64, i64, i64, i64, dp, dp,
+                                            ctypes.POINTER(ctypes.c_int32), dp]
+            lib.oracle_rollback.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _f64(a):
+    if a is None:
+        return None
+    if hasattr(a, "detach"):  # a torch tensor: widen exactly on the host
+        a = a.detach().to("cpu").double().numpy()
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.POINTER(ctypes.c_double))
+
+
+def default_threads() -> int:
+    return os.cpu_count() or 1
+
+
+def scan(x, dt, B, C, A, *, z=None, D=None, dt_bias=None, h0=None, b_rule=B_EULER,
+         want_h_all=False, nthreads=None):
+    """Run the layer core over [batch, L] and return (y, h_last, h_all or None).
+
+    x, dt, z: [batch, L, D]; B, C: [batch, L, N]; A: [D, N]; D, dt_bias: [D];
+    h0: [batch, D, N] or None (zeros). All outputs are float64.
+    """
+    x, dt, B, C, A = map(_f64, (x, dt, B, C, A))
+    z, D, dt_bias, h0 = map(_f64, (z, D, dt_bias, h0))
+    batch, L, Dn = x.shape
+    N = A.shape[1]
+    assert dt.shape == x.shape and B.shape == (batch, L, N) and C.shape == (batch, L, N)
+    assert A.shape == (Dn, N)
+    assert z is None or z.shape == x.shape
+    assert h0 is None or h0.shape == (batch, Dn, N)
+    y = np.empty((batch, L, Dn), dtype=np.float64)
+    h_last = np.empty((batch, Dn, N), dtype=np.float64)
+    h_all = np.empty((batch, L, Dn, N), dtype=np.float64) if want_h_all else None
+    rc = _load().oracle_scan(batch, L, Dn, N, _ptr(x), _ptr(z), _ptr(dt), _ptr(B), _ptr(C),
+                             _ptr(A), _ptr(D), _ptr(dt_bias), _ptr(h0), int(b_rule), _ptr(y),
+                             _ptr(h_last), _ptr(h_all), int(nthreads or default_threads()))
+    if rc != 0:
+        raise RuntimeError(f"oracle_scan failed ({rc})")
+    return y, h_last, h_all
+
+
+def step(state, x, dt, B, C, A, *, z=None, D=None, dt_bias=None, b_rule=B_EULER, nthreads=None):
+    """One recurrent decode step. x, dt, z: [batch, D]; B, C: [batch, N];
+    state: [batch, D, N]. Returns (y [batch, D], new_state)."""
+    x, dt, B, C, z = (None if a is None else _f64(a)[:, None] for a in (x, dt, B, C, z))
+    y, h, _ = scan(x, dt, B, C, A, z=z, D=D, dt_bias=dt_bias, h0=state, b_rule=b_rule,
+                   nthreads=nthreads)
+    return y[:, 0], h
+
+
+def rollback(h0, h_all, accept):
+    """State kept after accept[s] drafted bytes: h0[s] if accept[s] == 0, else
+    h_all[s, accept[s] - 1]. h_all: [batch, k, D, N]; h0: [batch, D, N] or None."""
+    h_all = _f64(h_all)
+    h0 = _f64(h0)
+    batch, k, Dn, N = h_all.shape
+    acc = np.ascontiguousarray(np.asarray(accept.cpu() if hasattr(accept, "cpu") else accept),
+                               dtype=np.int32)
+    out = np.empty((batch, Dn, N), dtype=np.float64)
+    rc = _load().oracle_rollback(batch, k, Dn, N, _ptr(h0), _ptr(h_all),
+                                 acc.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), _ptr(out))
+    if rc != 0:
+        raise RuntimeError("oracle_rollback: accept count out of [0, k]")
+    return out
