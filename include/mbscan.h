@@ -1,0 +1,157 @@
+/*
+ * mbscan.h - C ABI of the GB300 selective-scan layer core of MambaByte
+ * (arXiv 2401.13660).
+ *
+ * The layer core is the selective SSM of Section 2 (Eq. 1-3), discretised as
+ * in the appendix "Discretization and selection" (zero-order hold for A, the
+ * Euler rule Bbar = Delta*B that Mamba uses for B), followed by the output
+ * and gating rows of Table 6:
+ *
+ *   Delta_t = softplus(dt[b,t,d] + dt_bias[d])                   (Eq. 3)
+ *   h_t[n]  = exp(Delta_t * A[d,n]) * h_{t-1}[n]
+ *             + Delta_t * B[b,t,n] * x[b,t,d]                    (Eq. 2)
+ *   y[b,t,d] = (sum_n C[b,t,n] * h_t[n] + D[d] * x[b,t,d]) * silu(z[b,t,d])
+ *
+ * with one fp32 state vector h[b,d,0..N-1] per (batch row, channel). Every
+ * (b, d) channel is independent; the recurrence runs over t.
+ *
+ * Conventions shared by every entry point:
+ *  - All tensor pointers are DEVICE pointers (cudaMalloc / torch CUDA
+ *    tensors), row-major and contiguous, 16-byte aligned. The caller owns
+ *    every buffer; the library allocates nothing.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream). Every call is asynchronous on that stream.
+ *  - Argument errors are detected on the host before any launch and return
+ *    MB_ERR_INVALID_ARG or MB_ERR_UNSUPPORTED; nothing is launched then.
+ *    A failed launch returns MB_ERR_CUDA.
+ *  - Outputs must not alias inputs unless stated.
+ *  - Supported today: d_state == 16, dtype MB_F32 or MB_BF16,
+ *    d_inner % 8 == 0, batch*seqlen*d_inner < 2^31.
+ */
+#ifndef MBSCAN_H
+#define MBSCAN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MB_OK = 0,
+    MB_ERR_INVALID_ARG = 1,  /* null pointer, bad size, misalignment, aliasing */
+    MB_ERR_UNSUPPORTED = 2,  /* valid but not implemented (d_state, dtype)     */
+    MB_ERR_CUDA = 3,         /* a CUDA runtime call failed                       */
+    MB_ERR_TIMEOUT = 4       /* a bounded device-side wait gave up               */
+} mb_status;
+
+typedef enum { MB_F32 = 0, MB_BF16 = 1 } mb_dtype;
+
+/*
+ * Arguments of one selective-scan problem (Eq. 2-3 and Table 6).
+ *   batch    : independent sequences (>= 0)
+ *   seqlen   : time steps L (>= 0); 1 for mb_step
+ *   d_inner  : channels D = e * d_model (the SSM's input width)
+ *   d_state  : N = n_state, state size per channel (16 in MambaByte)
+ *   dtype    : element type of x, z, dt, B, C and y (mb_dtype)
+ *   x, z, dt : [batch, seqlen, d_inner], dtype. dt is the pre-softplus
+ *              timestep (W_Delta W_R x in Eq. 3). z is the gate input; NULL
+ *              means no gate (y = C.h + D x).
+ *   B, C     : [batch, seqlen, d_state], dtype (W_B x and W_C x in Eq. 3)
+ *   A        : [d_inner, d_state] fp32, the diagonal of A per channel
+ *   D        : [d_inner] fp32 skip weight; NULL means 0
+ *   dt_bias  : [d_inner] fp32 added to dt before softplus; NULL means 0
+ *   h0       : [batch, d_inner, d_state] fp32 initial state; NULL means 0
+ *   y        : [batch, seqlen, d_inner], dtype, output
+ */
+typedef struct {
+    int64_t batch, seqlen, d_inner, d_state;
+    int32_t dtype;
+    int32_t reserved;
+    const void *x, *z, *dt;
+    const void *B, *C;
+    const float *A;
+    const float *D;
+    const float *dt_bias;
+    const float *h0;
+    void *y;
+} mb_scan_args;
+
+/* Bytes of device workspace that mb_scan_prefill / mb_scan_verify need for
+ * `args` (a status block written by bounded device-side waits). The caller
+ * allocates it (256-byte aligned) and may reuse it across calls on one
+ * stream; calls that overlap on the GPU need distinct workspaces. Returns 0
+ * for invalid arguments. */
+size_t mb_workspace_size(const mb_scan_args *args);
+
+/*
+ * Prefill / training-forward scan (Section 2 "parallel scans": the whole span
+ * is available at once). Runs the layer core over all `seqlen` steps of every
+ * channel, writes y and, if h_last != NULL, the final state
+ * h_last[batch, d_inner, d_state] fp32 (the state MambaByte caches to resume
+ * generation). h_last may alias h0.
+ *   ws, ws_bytes : workspace of at least mb_workspace_size(args) bytes; it
+ *                  must start zeroed once after allocation and is left zeroed
+ *                  by every successful call.
+ */
+mb_status mb_scan_prefill(const mb_scan_args *args, float *h_last, void *ws, size_t ws_bytes,
+                          void *stream);
+
+/*
+ * Speculative-decoding verify (Section 3 "Speculative decoding through
+ * subword drafting" and Algorithm 1): resume from the cached verifier state
+ * h0 and scan the k = args->seqlen drafted bytes of each stream in one call,
+ * recording every per-position state:
+ *   h_all[b, j, d, n] = state after drafted byte j (j = 0..k-1), fp32,
+ *   shape [batch, k, d_inner, d_state]; y as in prefill.
+ * h_all must not alias h0.
+ */
+mb_status mb_scan_verify(const mb_scan_args *args, float *h_all, void *ws, size_t ws_bytes,
+                         void *stream);
+
+/*
+ * Rollback at the bifurcation (Algorithm 1: the verifier resumes from the
+ * state after the accepted drafted bytes). For every stream s,
+ *   h_out[s] = h0[s]                 if accept[s] == 0
+ *            = h_all[s, accept[s]-1] if 1 <= accept[s] <= k
+ * h0: [batch, d_inner, d_state] fp32 (NULL = zeros), h_all: [batch, k,
+ * d_inner, d_state] fp32, accept: [batch] int32 on the device, h_out:
+ * [batch, d_inner, d_state] fp32. h_out may alias h0 (not h_all). An accept
+ * count outside [0, k] is a caller error: that stream's h_out is left
+ * untouched and the first such stream index is recorded in the status block
+ * of `ws` when ws != NULL (read it with mb_check).
+ */
+mb_status mb_rollback(const float *h0, const float *h_all, const int32_t *accept, float *h_out,
+                      int64_t batch, int64_t k, int64_t d_inner, int64_t d_state, void *ws,
+                      void *stream);
+
+/*
+ * One recurrent decode step (Section 6.3: generation runs the recurrence
+ * directly, one byte per call). args->seqlen must be 1; args->h0 is ignored.
+ * `state` [batch, d_inner, d_state] fp32 is read and updated in place; y is
+ * [batch, 1, d_inner]. Used for the corrector loop of Algorithm 1 and for
+ * plain generation.
+ */
+mb_status mb_step(const mb_scan_args *args, float *state, void *stream);
+
+/*
+ * Read and clear the status block of a workspace (blocking: waits for
+ * `stream`). Returns MB_OK, or the first device-side error recorded by
+ * calls on that workspace since the last mb_check. If detail != NULL it
+ * receives an error-specific value (e.g. the first bad stream of
+ * mb_rollback), else -1.
+ */
+mb_status mb_check(void *ws, void *stream, int64_t *detail);
+
+/* Human-readable name of a status code (static string). */
+const char *mb_status_string(mb_status s);
+
+/* Library version, e.g. "mbscan 0.1.0 sm_103a". */
+const char *mb_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MBSCAN_H */

@@ -1,0 +1,70 @@
+// Device helpers shared by the selective-scan kernels (sm_103a).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "internal.h"
+
+namespace mbscan {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr unsigned kFull = 0xffffffffu;
+
+// 2^x on the SFU (MUFU.EX2), flushing subnormal results to zero.
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// Delta = softplus(v) = log(1 + e^v) (Eq. 3). Above v = 15 the correction
+// log1p(e^-v) < 3.1e-7 is below fp32 resolution of v and is dropped.
+__device__ __forceinline__ float softplus(float v) {
+    return v > 15.f ? v : log1pf(ex2(v * kLog2e));
+}
+
+// silu(z) = z * sigmoid(z), the Swish gate of the Mamba block. For z < -88
+// e^-z overflows to inf and the quotient is -0, the correctly rounded limit.
+__device__ __forceinline__ float silu(float z) {
+    return __fdividef(z, 1.f + ex2(-z * kLog2e));
+}
+
+// Element loads of the input dtype, widened to fp32.
+__device__ __forceinline__ float to_f32(float v) { return v; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+template <typename T> __device__ __forceinline__ T from_f32(float v);
+template <> __device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) {
+    return __float2bfloat16_rn(v);
+}
+
+template <typename T> __device__ __forceinline__ float ldg1(const T *p) { return to_f32(__ldg(p)); }
+
+// Four consecutive elements starting at p (8-byte aligned for bf16, 16 for fp32).
+__device__ __forceinline__ float4 ldg4(const float *p) { return __ldg(reinterpret_cast<const float4 *>(p)); }
+__device__ __forceinline__ float4 ldg4(const __nv_bfloat16 *p) {
+    uint2 u = __ldg(reinterpret_cast<const uint2 *>(p));
+    return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                       __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+}
+
+// Two consecutive elements starting at p (4-byte aligned for bf16, 8 for fp32).
+__device__ __forceinline__ float2 ldg2(const float *p) { return __ldg(reinterpret_cast<const float2 *>(p)); }
+__device__ __forceinline__ float2 ldg2(const __nv_bfloat16 *p) {
+    unsigned u = __ldg(reinterpret_cast<const unsigned *>(p));
+    return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
+}
+
+// Record the first device-side error of a call in the workspace status block.
+__device__ __forceinline__ void report(StatusBlock *sb, int code, long long detail) {
+    if (sb == nullptr) return;
+    if (atomicCAS(&sb->code, 0, code) == 0) {
+        sb->detail = detail;
+        __threadfence();
+    }
+}
+
+}  // namespace mbscan

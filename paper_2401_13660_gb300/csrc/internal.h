@@ -1,0 +1,38 @@
+// Internal launcher interface between the C ABI (mbscan_api.cu) and the
+// kernels. Plain C++ structs of device pointers and sizes; no torch types.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace mbscan {
+
+// Layout of the workspace status block (first bytes of `ws`).
+struct StatusBlock {
+    int code;        // 0 = ok, else an mb_status value
+    int pad;
+    long long detail;  // error-specific (first bad stream, ...), -1 when unset
+};
+constexpr size_t kStatusBytes = 256;
+
+// One selective-scan problem, validated by the API layer.
+struct ScanParams {
+    int64_t batch, seqlen, d_inner;  // d_state is fixed to 16
+    const void *x, *z, *dt, *B, *C;
+    const float *A, *D, *dt_bias, *h0;
+    void *y;
+    float *h_out;      // prefill: h_last (may be null); verify: h_all; step: state
+    StatusBlock *status;
+};
+
+constexpr int kDState = 16;
+
+// Launchers: return the cudaError_t of the launch.
+cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s);
+cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s);
+cudaError_t launch_step(const ScanParams &p, bool bf16, cudaStream_t s);
+cudaError_t launch_rollback(const float *h0, const float *h_all, const int32_t *accept,
+                            float *h_out, int64_t batch, int64_t k, int64_t d_inner,
+                            StatusBlock *status, cudaStream_t s);
+
+}  // namespace mbscan

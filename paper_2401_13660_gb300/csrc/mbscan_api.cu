@@ -1,0 +1,211 @@
+// C ABI of the selective-scan layer core: host-side validation, then one
+// kernel launch per call on the caller's stream. Declarations and the
+// contract of every entry point are in include/mbscan.h.
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string.h>
+
+#include "../../include/mbscan.h"
+#include "internal.h"
+
+using mbscan::ScanParams;
+using mbscan::StatusBlock;
+
+namespace {
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+struct Range {
+    uintptr_t lo, hi;
+};
+Range range_of(const void *p, int64_t bytes) {
+    uintptr_t a = reinterpret_cast<uintptr_t>(p);
+    return Range{a, a + (uintptr_t)(bytes > 0 ? bytes : 0)};
+}
+bool overlap(Range a, Range b) { return a.lo < b.hi && b.lo < a.hi && a.lo != a.hi && b.lo != b.hi; }
+
+// Products of sizes must stay far from int64 overflow and inside the
+// 32-bit element counts the kernels assume for token tensors.
+constexpr int64_t kMaxTokens = (int64_t)1 << 31;
+
+// Validate the common part of a scan problem; `need_seqlen1` for mb_step.
+mb_status check_args(const mb_scan_args *a, bool need_seqlen1) {
+    if (a == nullptr) return MB_ERR_INVALID_ARG;
+    if (a->batch < 0 || a->seqlen < 0 || a->d_inner < 0 || a->d_state < 0) return MB_ERR_INVALID_ARG;
+    if (a->dtype != MB_F32 && a->dtype != MB_BF16) return MB_ERR_INVALID_ARG;
+    if (need_seqlen1 && a->seqlen != 1) return MB_ERR_INVALID_ARG;
+    if (a->d_state != mbscan::kDState) return MB_ERR_UNSUPPORTED;
+    if (a->d_inner % 8 != 0) return MB_ERR_UNSUPPORTED;
+    if (a->batch > kMaxTokens || a->seqlen > kMaxTokens || a->d_inner > kMaxTokens)
+        return MB_ERR_INVALID_ARG;
+    const int64_t chans = a->batch * a->d_inner;
+    if (a->seqlen > 0 && chans > kMaxTokens / a->seqlen) return MB_ERR_INVALID_ARG;
+    if (chans > kMaxTokens / mbscan::kDState) return MB_ERR_INVALID_ARG;
+    const bool any_tokens = a->batch * a->seqlen * a->d_inner > 0;
+    const bool any_chan = chans > 0;
+    if (any_tokens && (!a->x || !a->dt || !a->B || !a->C || !a->y)) return MB_ERR_INVALID_ARG;
+    if (any_chan && !a->A) return MB_ERR_INVALID_ARG;
+    const void *ptrs[] = {a->x, a->z, a->dt, a->B, a->C, a->A, a->D, a->dt_bias, a->h0, a->y};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return MB_ERR_INVALID_ARG;
+    // y must not overlap any input.
+    const int64_t es = a->dtype == MB_BF16 ? 2 : 4;
+    const int64_t tok = a->batch * a->seqlen * a->d_inner * es;
+    const int64_t bc = a->batch * a->seqlen * a->d_state * es;
+    const Range ry = range_of(a->y, tok);
+    const Range ins[] = {range_of(a->x, tok), range_of(a->z, tok), range_of(a->dt, tok),
+                         range_of(a->B, bc), range_of(a->C, bc),
+                         range_of(a->A, a->d_inner * a->d_state * 4),
+                         range_of(a->D, a->d_inner * 4), range_of(a->dt_bias, a->d_inner * 4),
+                         range_of(a->h0, chans * a->d_state * 4)};
+    for (const Range &r : ins)
+        if (overlap(ry, r)) return MB_ERR_INVALID_ARG;
+    return MB_OK;
+}
+
+ScanParams to_params(const mb_scan_args *a, float *h_out, StatusBlock *status) {
+    ScanParams p;
+    p.batch = a->batch;
+    p.seqlen = a->seqlen;
+    p.d_inner = a->d_inner;
+    p.x = a->x; p.z = a->z; p.dt = a->dt; p.B = a->B; p.C = a->C;
+    p.A = a->A; p.D = a->D; p.dt_bias = a->dt_bias; p.h0 = a->h0;
+    p.y = a->y;
+    p.h_out = h_out;
+    p.status = status;
+    return p;
+}
+
+mb_status check_ws(const mb_scan_args *a, void *ws, size_t ws_bytes) {
+    const size_t need = mb_workspace_size(a);
+    if (need == 0) return MB_OK;
+    if (ws == nullptr || ws_bytes < need) return MB_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return MB_ERR_INVALID_ARG;
+    return MB_OK;
+}
+
+mb_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MB_OK : MB_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+size_t mb_workspace_size(const mb_scan_args *args) {
+    if (check_args(args, false) != MB_OK) return 0;
+    return mbscan::kStatusBytes;
+}
+
+mb_status mb_scan_prefill(const mb_scan_args *args, float *h_last, void *ws, size_t ws_bytes,
+                          void *stream) {
+    mb_status st = check_args(args, false);
+    if (st != MB_OK) return st;
+    if ((st = check_ws(args, ws, ws_bytes)) != MB_OK) return st;
+    const int64_t sbytes = args->batch * args->d_inner * args->d_state * 4;
+    if (h_last) {
+        if (!aligned16(h_last)) return MB_ERR_INVALID_ARG;
+        const Range rh = range_of(h_last, sbytes);
+        // h_last may be exactly h0 (in-place resume) but not partially overlap it.
+        if (args->h0 != h_last && overlap(rh, range_of(args->h0, sbytes))) return MB_ERR_INVALID_ARG;
+        const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
+        const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
+        if (overlap(rh, range_of(args->y, tok)) || overlap(rh, range_of(args->x, tok)) ||
+            overlap(rh, range_of(args->dt, tok)) || overlap(rh, range_of(args->z, tok)))
+            return MB_ERR_INVALID_ARG;
+    }
+    if (args->batch * args->d_inner == 0) return MB_OK;
+    ScanParams p = to_params(args, h_last, static_cast<StatusBlock *>(ws));
+    return from_cuda(mbscan::launch_prefill(p, args->dtype == MB_BF16, (cudaStream_t)stream));
+}
+
+mb_status mb_scan_verify(const mb_scan_args *args, float *h_all, void *ws, size_t ws_bytes,
+                         void *stream) {
+    mb_status st = check_args(args, false);
+    if (st != MB_OK) return st;
+    if ((st = check_ws(args, ws, ws_bytes)) != MB_OK) return st;
+    const int64_t n_all = args->batch * args->seqlen * args->d_inner * args->d_state;
+    if (n_all > 0) {
+        if (h_all == nullptr || !aligned16(h_all)) return MB_ERR_INVALID_ARG;
+        const Range ra = range_of(h_all, n_all * 4);
+        const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
+        const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
+        if (overlap(ra, range_of(args->h0, args->batch * args->d_inner * args->d_state * 4)) ||
+            overlap(ra, range_of(args->y, tok)) || overlap(ra, range_of(args->x, tok)) ||
+            overlap(ra, range_of(args->dt, tok)) || overlap(ra, range_of(args->z, tok)))
+            return MB_ERR_INVALID_ARG;
+    }
+    if (n_all == 0) return MB_OK;
+    ScanParams p = to_params(args, h_all, static_cast<StatusBlock *>(ws));
+    return from_cuda(mbscan::launch_verify(p, args->dtype == MB_BF16, (cudaStream_t)stream));
+}
+
+mb_status mb_rollback(const float *h0, const float *h_all, const int32_t *accept, float *h_out,
+                      int64_t batch, int64_t k, int64_t d_inner, int64_t d_state, void *ws,
+                      void *stream) {
+    if (batch < 0 || k < 0 || d_inner < 0 || d_state < 0) return MB_ERR_INVALID_ARG;
+    if (d_state != mbscan::kDState) return MB_ERR_UNSUPPORTED;
+    if (batch > kMaxTokens || k > kMaxTokens || d_inner > kMaxTokens) return MB_ERR_INVALID_ARG;
+    const int64_t per = d_inner * d_state;
+    if (batch > 0 && per > 0 && k > 0 && batch * k > kMaxTokens * 16 / per) return MB_ERR_INVALID_ARG;
+    if (batch * per == 0) return MB_OK;
+    if (!accept || !h_out || (k > 0 && !h_all)) return MB_ERR_INVALID_ARG;
+    if (!aligned16(h_out) || (h0 && !aligned16(h0)) || (h_all && !aligned16(h_all)) ||
+        (reinterpret_cast<uintptr_t>(accept) & 3u))
+        return MB_ERR_INVALID_ARG;
+    if (ws && (reinterpret_cast<uintptr_t>(ws) & 255u)) return MB_ERR_INVALID_ARG;
+    const Range ro = range_of(h_out, batch * per * 4);
+    if (overlap(ro, range_of(h_all, batch * k * per * 4))) return MB_ERR_INVALID_ARG;
+    if (h0 && h0 != h_out && overlap(ro, range_of(h0, batch * per * 4))) return MB_ERR_INVALID_ARG;
+    if (overlap(ro, range_of(accept, batch * 4))) return MB_ERR_INVALID_ARG;
+    return from_cuda(mbscan::launch_rollback(h0, h_all, accept, h_out, batch, k, d_inner,
+                                             static_cast<StatusBlock *>(ws), (cudaStream_t)stream));
+}
+
+mb_status mb_step(const mb_scan_args *args, float *state, void *stream) {
+    mb_status st = check_args(args, true);
+    if (st != MB_OK) return st;
+    const int64_t chans = args->batch * args->d_inner;
+    if (chans == 0) return MB_OK;
+    if (state == nullptr || !aligned16(state)) return MB_ERR_INVALID_ARG;
+    const Range rs = range_of(state, chans * args->d_state * 4);
+    const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
+    const int64_t tok = chans * es;
+    const Range others[] = {range_of(args->y, tok), range_of(args->x, tok), range_of(args->z, tok),
+                            range_of(args->dt, tok), range_of(args->B, args->batch * args->d_state * es),
+                            range_of(args->C, args->batch * args->d_state * es),
+                            range_of(args->A, args->d_inner * args->d_state * 4)};
+    for (const Range &r : others)
+        if (overlap(rs, r)) return MB_ERR_INVALID_ARG;
+    ScanParams p = to_params(args, state, nullptr);
+    p.h0 = nullptr;
+    return from_cuda(mbscan::launch_step(p, args->dtype == MB_BF16, (cudaStream_t)stream));
+}
+
+mb_status mb_check(void *ws, void *stream, int64_t *detail) {
+    if (detail) *detail = -1;
+    if (ws == nullptr) return MB_ERR_INVALID_ARG;
+    StatusBlock host;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cudaMemcpyAsync(&host, ws, sizeof(host), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return MB_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return MB_ERR_CUDA;
+    if (host.code == MB_OK) return MB_OK;
+    if (cudaMemsetAsync(ws, 0, sizeof(StatusBlock), s) != cudaSuccess) return MB_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return MB_ERR_CUDA;
+    if (detail) *detail = host.detail;
+    return (mb_status)host.code;
+}
+
+const char *mb_status_string(mb_status s) {
+    switch (s) {
+        case MB_OK: return "MB_OK";
+        case MB_ERR_INVALID_ARG: return "MB_ERR_INVALID_ARG";
+        case MB_ERR_UNSUPPORTED: return "MB_ERR_UNSUPPORTED";
+        case MB_ERR_CUDA: return "MB_ERR_CUDA";
+        case MB_ERR_TIMEOUT: return "MB_ERR_TIMEOUT";
+    }
+    return "MB_UNKNOWN_STATUS";
+}
+
+const char *mb_version(void) { return "mbscan 0.1.0 sm_103a"; }
+
+}  // extern "C"

@@ -1,0 +1,205 @@
+"""Python binding of libmbscan.so (argument marshalling only).
+
+Each function has the name of the C entry point it calls (include/mbscan.h)
+and takes torch CUDA tensors in place of device pointers. Every step of the
+layer core runs in the library's kernels; this module only checks tensor
+shapes/dtypes/devices, fills the C argument struct and forwards the call on
+the current torch CUDA stream (or the stream given). There is no fallback: if
+the library cannot be loaded, importing the functions raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+_lock = threading.Lock()
+_lib = None
+
+MB_OK, MB_ERR_INVALID_ARG, MB_ERR_UNSUPPORTED, MB_ERR_CUDA, MB_ERR_TIMEOUT = range(5)
+MB_F32, MB_BF16 = 0, 1
+_DTYPES = {torch.float32: MB_F32, torch.bfloat16: MB_BF16}
+
+
+class MbError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {mb_status_string(status)}")
+
+
+class mb_scan_args(ctypes.Structure):
+    _fields_ = [
+        ("batch", ctypes.c_int64), ("seqlen", ctypes.c_int64),
+        ("d_inner", ctypes.c_int64), ("d_state", ctypes.c_int64),
+        ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("x", ctypes.c_void_p), ("z", ctypes.c_void_p), ("dt", ctypes.c_void_p),
+        ("B", ctypes.c_void_p), ("C", ctypes.c_void_p),
+        ("A", ctypes.c_void_p), ("D", ctypes.c_void_p), ("dt_bias", ctypes.c_void_p),
+        ("h0", ctypes.c_void_p), ("y", ctypes.c_void_p),
+    ]
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
+    """Load libmbscan.so (building it first if it is missing or stale)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = _build.build() if build_if_needed else _build.LIB
+            if not os.path.exists(path):
+                raise RuntimeError(f"libmbscan.so not found at {path}; run build() first")
+            lib = ctypes.CDLL(path)
+            vp, i64, sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_size_t
+            ap = ctypes.POINTER(mb_scan_args)
+            lib.mb_workspace_size.argtypes = [ap]
+            lib.mb_workspace_size.restype = sz
+            lib.mb_scan_prefill.argtypes = [ap, vp, vp, sz, vp]
+            lib.mb_scan_verify.argtypes = [ap, vp, vp, sz, vp]
+            lib.mb_rollback.argtypes = [vp, vp, vp, vp, i64, i64, i64, i64, vp, vp]
+            lib.mb_step.argtypes = [ap, vp, vp]
+            lib.mb_check.argtypes = [vp, vp, ctypes.POINTER(i64)]
+            for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_check"):
+                getattr(lib, f).restype = ctypes.c_int
+            lib.mb_status_string.argtypes = [ctypes.c_int]
+            lib.mb_status_string.restype = ctypes.c_char_p
+            lib.mb_version.argtypes = []
+            lib.mb_version.restype = ctypes.c_char_p
+            _lib = lib
+    return _lib
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _need(t, name, dtype=None, shape=None, device=None):
+    if t is None:
+        return
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name}: dtype {t.dtype}, expected {dtype}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name}: shape {tuple(t.shape)}, expected {tuple(shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+
+
+def make_args(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None) -> mb_scan_args:
+    """Fill mb_scan_args from tensors. x, dt, z, y: [batch, L, d_inner];
+    B, C: [batch, L, d_state] (all one dtype, fp32 or bf16); A: [d_inner,
+    d_state], D, dt_bias: [d_inner], h0: [batch, d_inner, d_state] (fp32)."""
+    if x.dtype not in _DTYPES:
+        raise TypeError(f"unsupported input dtype {x.dtype}")
+    batch, L, Dn = x.shape
+    N = A.shape[1]
+    dev = x.device
+    for name, t in (("x", x), ("dt", dt), ("z", z), ("y", y)):
+        _need(t, name, x.dtype, (batch, L, Dn), dev)
+    for name, t in (("B", B), ("C", C)):
+        _need(t, name, x.dtype, (batch, L, N), dev)
+    _need(A, "A", torch.float32, (Dn, N), dev)
+    _need(D, "D", torch.float32, (Dn,), dev)
+    _need(dt_bias, "dt_bias", torch.float32, (Dn,), dev)
+    _need(h0, "h0", torch.float32, (batch, Dn, N), dev)
+    a = mb_scan_args()
+    a.batch, a.seqlen, a.d_inner, a.d_state = batch, L, Dn, N
+    a.dtype = _DTYPES[x.dtype]
+    a.x, a.z, a.dt, a.B, a.C = (t.data_ptr() if t is not None else None for t in (x, z, dt, B, C))
+    a.A, a.D, a.dt_bias, a.h0 = (t.data_ptr() if t is not None else None for t in (A, D, dt_bias, h0))
+    a.y = y.data_ptr()
+    return a
+
+
+def _check(rc, where):
+    if rc != MB_OK:
+        raise MbError(rc, where)
+
+
+def mb_status_string(status: int) -> str:
+    return load_library().mb_status_string(int(status)).decode()
+
+
+def mb_version() -> str:
+    return load_library().mb_version().decode()
+
+
+def mb_workspace_size(args: mb_scan_args) -> int:
+    return int(load_library().mb_workspace_size(ctypes.byref(args)))
+
+
+def new_workspace(args: mb_scan_args, device) -> torch.Tensor:
+    """Zeroed workspace tensor for `args` (uint8, 256-byte aligned by torch)."""
+    n = max(mb_workspace_size(args), 256)
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def mb_scan_prefill(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None, h_last=None,
+                    ws=None, stream=None):
+    """Prefill scan: writes y and (if given) h_last [batch, d_inner, d_state]."""
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0)
+    _need(h_last, "h_last", torch.float32, (a.batch, a.d_inner, a.d_state), x.device)
+    if ws is None:
+        ws = new_workspace(a, x.device)
+    rc = load_library().mb_scan_prefill(ctypes.byref(a), _ptr(h_last), _ptr(ws), ws.numel(),
+                                        _stream(stream))
+    _check(rc, "mb_scan_prefill")
+    return y, h_last
+
+
+def mb_scan_verify(x, dt, B, C, A, y, h_all, *, z=None, D=None, dt_bias=None, h0=None, ws=None,
+                   stream=None):
+    """Verify scan of k = x.shape[1] drafted bytes: y and h_all [batch, k, d_inner, d_state]."""
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0)
+    _need(h_all, "h_all", torch.float32, (a.batch, a.seqlen, a.d_inner, a.d_state), x.device)
+    if ws is None:
+        ws = new_workspace(a, x.device)
+    rc = load_library().mb_scan_verify(ctypes.byref(a), _ptr(h_all), _ptr(ws), ws.numel(),
+                                       _stream(stream))
+    _check(rc, "mb_scan_verify")
+    return y, h_all
+
+
+def mb_rollback(h0, h_all, accept, h_out, *, ws=None, stream=None):
+    """h_out[s] = h0[s] if accept[s] == 0 else h_all[s, accept[s]-1]."""
+    batch, k, Dn, N = h_all.shape
+    _need(h_all, "h_all", torch.float32)
+    _need(h0, "h0", torch.float32, (batch, Dn, N), h_all.device)
+    _need(h_out, "h_out", torch.float32, (batch, Dn, N), h_all.device)
+    _need(accept, "accept", torch.int32, (batch,), h_all.device)
+    rc = load_library().mb_rollback(_ptr(h0), _ptr(h_all), _ptr(accept), _ptr(h_out), batch, k,
+                                    Dn, N, _ptr(ws), _stream(stream))
+    _check(rc, "mb_rollback")
+    return h_out
+
+
+def mb_step(x, dt, B, C, A, y, state, *, z=None, D=None, dt_bias=None, stream=None):
+    """One decode step: x, dt, z, y [batch, 1, d_inner]; B, C [batch, 1, d_state];
+    state [batch, d_inner, d_state] updated in place."""
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias)
+    _need(state, "state", torch.float32, (a.batch, a.d_inner, a.d_state), x.device)
+    rc = load_library().mb_step(ctypes.byref(a), _ptr(state), _stream(stream))
+    _check(rc, "mb_step")
+    return y, state
+
+
+def mb_check(ws, stream=None):
+    """Read and clear the workspace status block: (status, detail)."""
+    detail = ctypes.c_int64(-1)
+    rc = load_library().mb_check(_ptr(ws), _stream(stream), ctypes.byref(detail))
+    return int(rc), int(detail.value)

@@ -1,0 +1,54 @@
+"""Helpers shared by the parity tests: the error metric and oracle calls on
+the same seeded tensors that the CUDA path receives."""
+import numpy as np
+import torch
+
+import oracle
+
+# Tolerances on err = max |g - r| / max(|r|, rms(r)) per output tensor: the
+# state is fp32 in both cases; bf16 inputs/outputs add the bf16 rounding of y.
+TOL = {"f32": 1e-4, "bf16": 2e-2}
+
+
+def rel_err(got, ref) -> float:
+    """max_i |g_i - r_i| / max(|r_i|, rms(r)); 0 for empty tensors."""
+    g = got.detach().cpu().double().numpy() if isinstance(got, torch.Tensor) else np.asarray(got, dtype=np.float64)
+    r = np.asarray(ref, dtype=np.float64)
+    assert g.shape == r.shape, (g.shape, r.shape)
+    if r.size == 0:
+        return 0.0
+    rms = float(np.sqrt(np.mean(r * r)))
+    floor = np.maximum(np.abs(r), rms if rms > 0 else 1e-30)
+    return float(np.max(np.abs(g - r) / floor))
+
+
+def to_np(t):
+    return None if t is None else t.detach().cpu().double().numpy()
+
+
+def oracle_scan(inp, want_h_all=False, nthreads=None):
+    """Oracle over a whole input dict from paper_2401_13660_gb300.inputs."""
+    return oracle.scan(to_np(inp["x"]), to_np(inp["dt"]), to_np(inp["B"]), to_np(inp["C"]),
+                       to_np(inp["A"]), z=to_np(inp.get("z")), D=to_np(inp.get("D")),
+                       dt_bias=to_np(inp.get("dt_bias")), h0=to_np(inp.get("h0")),
+                       want_h_all=want_h_all, nthreads=nthreads)
+
+
+def oracle_channels(inp, rows, chans, nthreads=None):
+    """Oracle on the sub-problem of batch rows `rows` and channels `chans`
+    (channels are independent, so slicing them out is exact)."""
+    rows = torch.as_tensor(rows)
+    chans = torch.as_tensor(chans)
+
+    def tok(t):
+        return None if t is None else to_np(t.index_select(0, rows.to(t.device))[:, :, chans.to(t.device)])
+
+    def bc(t):
+        return to_np(t.index_select(0, rows.to(t.device)))
+
+    h0 = inp.get("h0")
+    h0s = None if h0 is None else to_np(h0.index_select(0, rows.to(h0.device))[:, chans.to(h0.device)])
+    pick = lambda t: None if t is None else to_np(t[chans.to(t.device)])
+    return oracle.scan(tok(inp["x"]), tok(inp["dt"]), bc(inp["B"]), bc(inp["C"]), pick(inp["A"]),
+                       z=tok(inp.get("z")), D=pick(inp.get("D")), dt_bias=pick(inp.get("dt_bias")),
+                       h0=h0s, nthreads=nthreads)

@@ -1,0 +1,148 @@
+"""CPU checks of the C ABI: the library loads, exports every entry point that
+include/mbscan.h declares, and rejects bad arguments on the host before any
+launch (so these run without a GPU: no call below reaches the device)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2401_13660_gb300 import mbscan as mb
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "mbscan.h")
+
+FAKE = 1 << 40  # an aligned, never-dereferenced stand-in for a device address
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(mb_[a-z_]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_workspace_size",
+              "mb_check", "mb_status_string", "mb_version"):
+        assert f in names
+
+
+def test_library_exports_every_declared_symbol():
+    lib = mb.load_library()
+    for f in declared_functions():
+        assert hasattr(lib, f), f
+    out = subprocess.run(["nm", "-D", "--defined-only", mb.library_path()], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r" T (mb_[a-z_]+)$", out, flags=re.M))
+    assert set(declared_functions()) <= exported
+
+
+def test_status_strings_and_version():
+    assert mb.mb_status_string(0) == "MB_OK"
+    assert mb.mb_status_string(2) == "MB_ERR_UNSUPPORTED"
+    assert mb.mb_status_string(99) == "MB_UNKNOWN_STATUS"
+    assert "sm_103a" in mb.mb_version()
+
+
+def _args(batch=2, L=8, Dn=64, N=16, dtype=mb.MB_BF16, **kw):
+    a = mb.mb_scan_args()
+    a.batch, a.seqlen, a.d_inner, a.d_state, a.dtype = batch, L, Dn, N, dtype
+    base = FAKE
+    for i, f in enumerate(("x", "z", "dt", "B", "C", "A", "D", "dt_bias", "h0", "y")):
+        setattr(a, f, base + i * (1 << 32))
+    for k, v in kw.items():
+        setattr(a, k, v)
+    return a
+
+
+def _call(name, a, *extra):
+    lib = mb.load_library()
+    return getattr(lib, name)(ctypes.byref(a), *extra)
+
+
+def _prefill(a, h_last=None, ws=FAKE + (200 << 32), ws_bytes=256):
+    return _call("mb_scan_prefill", a, h_last, ws, ws_bytes, None)
+
+
+def test_workspace_size():
+    lib = mb.load_library()
+    assert lib.mb_workspace_size(ctypes.byref(_args())) == 256
+    assert lib.mb_workspace_size(ctypes.byref(_args(N=8))) == 0
+    assert lib.mb_workspace_size(None) == 0
+
+
+@pytest.mark.parametrize("bad, want", [
+    (dict(N=8), mb.MB_ERR_UNSUPPORTED),
+    (dict(Dn=60), mb.MB_ERR_UNSUPPORTED),
+    (dict(dtype=7), mb.MB_ERR_INVALID_ARG),
+    (dict(batch=-1), mb.MB_ERR_INVALID_ARG),
+    (dict(L=-3), mb.MB_ERR_INVALID_ARG),
+    (dict(x=None), mb.MB_ERR_INVALID_ARG),
+    (dict(A=None), mb.MB_ERR_INVALID_ARG),
+    (dict(y=None), mb.MB_ERR_INVALID_ARG),
+    (dict(dt=FAKE + 8), mb.MB_ERR_INVALID_ARG),          # misaligned
+    (dict(L=1 << 20, Dn=1 << 12, batch=1 << 10), mb.MB_ERR_INVALID_ARG),  # too many tokens
+])
+def test_prefill_rejects_bad_args(bad, want):
+    kw = {}
+    for k in ("batch", "L", "Dn", "N", "dtype"):
+        if k in bad:
+            kw[k] = bad.pop(k)
+    a = _args(**kw)
+    for k, v in bad.items():
+        setattr(a, k, v)
+    assert _prefill(a) == want
+
+
+def test_prefill_rejects_aliasing_and_missing_workspace():
+    a = _args()
+    a.y = a.x + 64                                   # y overlaps x
+    assert _prefill(a) == mb.MB_ERR_INVALID_ARG
+    a = _args()
+    assert _prefill(a, ws=None) == mb.MB_ERR_INVALID_ARG
+    assert _prefill(a, ws_bytes=16) == mb.MB_ERR_INVALID_ARG
+    assert _prefill(a, ws=FAKE + (200 << 32) + 16) == mb.MB_ERR_INVALID_ARG   # ws not 256-aligned
+    assert _prefill(a, h_last=a.h0 + 16) == mb.MB_ERR_INVALID_ARG           # partial overlap with h0
+    assert _prefill(a, h_last=a.y) == mb.MB_ERR_INVALID_ARG
+
+
+def test_zero_sized_calls_launch_nothing():
+    lib = mb.load_library()
+    assert _prefill(_args(batch=0)) == mb.MB_OK
+    assert _call("mb_scan_verify", _args(L=0), None, FAKE + (200 << 32), 256, None) == mb.MB_OK
+    assert _call("mb_step", _args(batch=0, L=1), None, None) == mb.MB_OK
+    assert lib.mb_rollback(None, None, None, None, 0, 16, 64, 16, None, None) == mb.MB_OK
+
+
+def test_verify_and_step_checks():
+    a = _args(L=16)
+    assert _call("mb_scan_verify", a, None, FAKE + (200 << 32), 256, None) == mb.MB_ERR_INVALID_ARG
+    assert _call("mb_scan_verify", a, a.h0, FAKE + (200 << 32), 256, None) == mb.MB_ERR_INVALID_ARG
+    s = _args(L=2)
+    assert _call("mb_step", s, FAKE + (210 << 32), None) == mb.MB_ERR_INVALID_ARG   # seqlen != 1
+    s = _args(L=1)
+    assert _call("mb_step", s, None, None) == mb.MB_ERR_INVALID_ARG
+    assert _call("mb_step", s, s.x, None) == mb.MB_ERR_INVALID_ARG               # state aliases x
+
+
+def test_rollback_checks():
+    lib = mb.load_library()
+    h0, h_all, acc, out = FAKE, FAKE + (1 << 34), FAKE + (2 << 34), FAKE + (3 << 34)
+    assert lib.mb_rollback(h0, h_all, acc, out, 4, 16, 64, 8, None, None) == mb.MB_ERR_UNSUPPORTED
+    assert lib.mb_rollback(h0, h_all, None, out, 4, 16, 64, 16, None, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_rollback(h0, h_all, acc, h_all + 64, 4, 16, 64, 16, None, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_rollback(h0, h_all, acc + 2, out, 4, 16, 64, 16, None, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_rollback(h0, h_all, acc, out, -1, 16, 64, 16, None, None) == mb.MB_ERR_INVALID_ARG
+
+
+def test_binding_rejects_cpu_shape_errors():
+    import torch
+    x = torch.zeros(1, 4, 8, dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        mb.make_args(x, x, torch.zeros(1, 4, 16, dtype=torch.bfloat16),
+                     torch.zeros(1, 4, 16, dtype=torch.bfloat16), torch.zeros(8, 16),
+                     torch.zeros(1, 4, 9, dtype=torch.bfloat16))
+    with pytest.raises(TypeError):
+        mb.make_args(x.float(), x, x, x, torch.zeros(8, 16), x)
