@@ -18,13 +18,15 @@ import sys
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
-BUILD = os.path.join(HERE, "_build")
+BUILD = os.environ.get("MBSCAN_BUILD_DIR") or os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libmbscan.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2",
               "--expt-relaxed-constexpr", "-I", INCLUDE]
+# Extra nvcc flags (e.g. -D tuning macros) for builds into MBSCAN_BUILD_DIR.
+NVCC_FLAGS += os.environ.get("MBSCAN_NVCC_FLAGS", "").split()
 
 
 def nvcc() -> str:

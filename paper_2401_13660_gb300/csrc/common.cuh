@@ -19,10 +19,26 @@ __device__ __forceinline__ float ex2(float x) {
     return y;
 }
 
-// Delta = softplus(v) = log(1 + e^v) (Eq. 3). Above v = 15 the correction
-// log1p(e^-v) < 3.1e-7 is below fp32 resolution of v and is dropped.
+constexpr float kLn2 = 0.6931471805599453f;
+
+// log2(x) on the SFU (MUFU.LG2).
+__device__ __forceinline__ float lg2(float x) {
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// Delta = softplus(v) = log(1 + e^v) (Eq. 3), with u = e^v from the SFU:
+//  * u < 2^-5: log1p(u) by its Taylor series to u^3 (truncation < 8e-6 relative);
+//  * otherwise: ln 2 * log2(1 + u) on the SFU, where 1 + u >= 1.03 carries no
+//    cancellation (relative error < 1e-5 at the switch point, falling above);
+//  * v > 15: v itself (the dropped log1p(e^-v) < 3.1e-7 is below fp32 resolution).
 __device__ __forceinline__ float softplus(float v) {
-    return v > 15.f ? v : log1pf(ex2(v * kLog2e));
+    const float u = ex2(v * kLog2e);
+    const float series = u * fmaf(u, fmaf(u, 0.33333334f, -0.5f), 1.f);
+    const float logw = lg2(1.f + u) * kLn2;
+    const float r = u < 0.03125f ? series : logw;
+    return v > 15.f ? v : r;
 }
 
 // silu(z) = z * sigmoid(z), the Swish gate of the Mamba block. For z < -88

@@ -1,176 +1,146 @@
 // Decode-side kernels of the selective-scan layer core: the batched
-// single-byte recurrent step, the speculative-decoding verify scan that keeps
-// every per-position state, and the rollback gather (MambaByte Section 3,
-// Section 6.3 and Algorithm 1).
+// single-byte recurrent step and the rollback gather of speculative decoding
+// (MambaByte Section 6.3 and Algorithm 1). The verify scan shares the prefill
+// kernel (prefill.cu).
 //
-// All three are HBM-streaming kernels: a (batch row, channel) pair owns 16
-// fp32 states (64 contiguous bytes). Four lanes share one channel, each lane
-// holding 4 states in one float4, so that a warp moves 512 contiguous bytes of
-// state per instruction. The channel's scalars (dt, x, z) are broadcast to the
-// four lanes; C.h is reduced over the four lanes with two xor-shuffles.
+// Both are HBM-streaming kernels. A (batch row, channel) pair owns 16 fp32
+// states (64 contiguous bytes). In the step kernel four lanes share a channel,
+// each holding 4 states in one float4, so a warp moves 512 contiguous bytes
+// of state per instruction; each lane group serves kSlots channels so that
+// every lane has kSlots independent 16-byte state loads in flight.
 #include "common.cuh"
+#include "tma.cuh"
 
 namespace mbscan {
 namespace {
 
-constexpr int kThreads = 256;         // 64 channels per CTA per channel slot
-constexpr int kChanPerCta = kThreads / 4;
+constexpr int kStepThreads = 256;
+constexpr int kSlots = 4;                                       // channels per lane group
+constexpr int kStepChPerWarp = 8 * kSlots;                      // 32
+constexpr int kStepChPerCta = kStepChPerWarp * (kStepThreads / 32);  // 256
 
-// One time step of one channel on one lane (states 4q..4q+3). Returns this
-// lane's share of C.h.
-__device__ __forceinline__ float lane_update(float4 &h, const float4 a2, float delta, float dx,
-                                            const float4 b, const float4 c) {
-    h.x = fmaf(ex2(delta * a2.x), h.x, b.x * dx);
-    h.y = fmaf(ex2(delta * a2.y), h.y, b.y * dx);
-    h.z = fmaf(ex2(delta * a2.z), h.z, b.z * dx);
-    h.w = fmaf(ex2(delta * a2.w), h.w, b.w * dx);
-    return fmaf(c.x, h.x, fmaf(c.y, h.y, fmaf(c.z, h.z, c.w * h.w)));
+// Lane q of a 4-lane group holds the group's shares part[0..3] (one per
+// slot); return the full 4-lane sum of slot q (two shuffle rounds).
+__device__ __forceinline__ float reduce_slots(const float (&part)[4], int q) {
+    const bool hi = (q & 2) != 0;
+    float k0 = hi ? part[2] : part[0], k1 = hi ? part[3] : part[1];
+    const float s0 = hi ? part[0] : part[2], s1 = hi ? part[1] : part[3];
+    k0 += __shfl_xor_sync(kFull, s0, 2);
+    k1 += __shfl_xor_sync(kFull, s1, 2);
+    const bool odd = (q & 1) != 0;
+    const float keep = odd ? k1 : k0, send = odd ? k0 : k1;
+    return keep + __shfl_xor_sync(kFull, send, 1);
 }
 
 // ---------------------------------------------------------------------------
-// mb_step: state[b, d, :] <- one recurrence step; y[b, 0, d]. CPT channels per
-// thread (strided by kChanPerCta) keep several 16-byte state loads in flight.
-template <typename T, int CPT>
-__global__ void __launch_bounds__(kThreads) step_kernel(ScanParams p) {
-    const int q = threadIdx.x & 3;
-    const int64_t nchan = p.batch * p.d_inner;
-    const int64_t base = (int64_t)blockIdx.x * (kChanPerCta * CPT) + (threadIdx.x >> 2);
+// mb_step: state[b, d, :] <- one recurrence step (Eq. 2 with L = 1), y[b, 0, d].
+// Lane (g, q) of a warp: slot j covers channel wbase + 8 j + g, states 4q..4q+3.
+// The lane computes the channel scalars (Delta, Delta*x, D*x, silu z) only for
+// slot q and hands Delta, Delta*x to its group by shuffle; after the 4-lane
+// reduction it also owns slot q's output.
+template <typename T>
+__global__ void __launch_bounds__(kStepThreads, 4) step_kernel(ScanParams p) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int g = lane >> 2, q = lane & 3;
+    const int64_t D = p.d_inner;
+    const int64_t nchan = p.batch * D;
+    const int64_t wbase = (int64_t)blockIdx.x * kStepChPerCta + warp * kStepChPerWarp;
     const T *x = static_cast<const T *>(p.x);
     const T *z = static_cast<const T *>(p.z);
     const T *dt = static_cast<const T *>(p.dt);
     const T *Bm = static_cast<const T *>(p.B);
     const T *Cm = static_cast<const T *>(p.C);
-    T *y = static_cast<T *>(p.y);
+    float4 *state = reinterpret_cast<float4 *>(p.h_out);
 
-    float4 h[CPT];
-    bool ok[CPT];
+    float4 h[kSlots];
 #pragma unroll
-    for (int j = 0; j < CPT; ++j) {
-        const int64_t ch = base + (int64_t)j * kChanPerCta;
-        ok[j] = ch < nchan;
-        h[j] = ok[j] ? __ldcs(reinterpret_cast<const float4 *>(p.h_out + ch * kDState) + q)
-                     : make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int j = 0; j < kSlots; ++j) {
+        const int64_t ch = wbase + 8 * j + g;
+        h[j] = ch < nchan ? __ldcs(state + ch * (kDState / 4) + q) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
+
+    // channel scalars of slot q
+    const int64_t mc = wbase + 8 * q + g;
+    const bool mok = mc < nchan;
+    const int64_t md = mok ? mc % D : 0;
+    float delta = 0.f, gx = 0.f, xd = 0.f, sz = 1.f;
+    if (mok) {
+        const float xv = ldg1(x + mc);
+        delta = softplus(ldg1(dt + mc) + (p.dt_bias ? __ldg(p.dt_bias + md) : 0.f));
+        gx = delta * xv;
+        xd = (p.D ? __ldg(p.D + md) : 0.f) * xv;
+        if (z) sz = silu(ldg1(z + mc));
+    }
+
+    float part[kSlots];
 #pragma unroll
-    for (int j = 0; j < CPT; ++j) {
-        const int64_t ch = base + (int64_t)j * kChanPerCta;
-        const int64_t b = ok[j] ? ch / p.d_inner : 0;
-        const int64_t d = ok[j] ? ch - b * p.d_inner : 0;
-        const int64_t i = ok[j] ? ch : 0;  // [b, 0, d] with seqlen 1
-        const float xv = ldg1(x + i);
-        const float v = ldg1(dt + i) + (p.dt_bias ? __ldg(p.dt_bias + d) : 0.f);
-        const float delta = softplus(v);
-        float4 a2 = ldg4(p.A + d * kDState + 4 * q);
-        a2.x *= kLog2e; a2.y *= kLog2e; a2.z *= kLog2e; a2.w *= kLog2e;
+    for (int j = 0; j < kSlots; ++j) {
+        const int64_t ch = wbase + 8 * j + g;
+        const int64_t cch = ch < nchan ? ch : 0;
+        const int64_t b = cch / D, d = cch - b * D;
+        const float dj = __shfl_sync(kFull, delta, 4 * g + j);
+        const float gj = __shfl_sync(kFull, gx, 4 * g + j);
+        const float4 av = ldg4(p.A + d * kDState + 4 * q);
         const float4 bv = ldg4(Bm + b * kDState + 4 * q);
         const float4 cv = ldg4(Cm + b * kDState + 4 * q);
-        float part = lane_update(h[j], a2, delta, delta * xv, bv, cv);
-        part += __shfl_xor_sync(kFull, part, 1);
-        part += __shfl_xor_sync(kFull, part, 2);
-        if (ok[j]) {
-            __stcs(reinterpret_cast<float4 *>(p.h_out + ch * kDState) + q, h[j]);
-            if (q == 0) {
-                float out = part + (p.D ? __ldg(p.D + d) : 0.f) * xv;
-                if (z) out *= silu(ldg1(z + i));
-                y[i] = from_f32<T>(out);
-            }
-        }
+        float2 h01 = make_float2(h[j].x, h[j].y), h23 = make_float2(h[j].z, h[j].w);
+        const float2 dd = make_float2(dj, dj), gg = make_float2(gj, gj);
+        const float2 e01 = mul2(dd, make_float2(av.x * kLog2e, av.y * kLog2e));
+        const float2 e23 = mul2(dd, make_float2(av.z * kLog2e, av.w * kLog2e));
+        h01 = fma2(make_float2(ex2(e01.x), ex2(e01.y)), h01, mul2(make_float2(bv.x, bv.y), gg));
+        h23 = fma2(make_float2(ex2(e23.x), ex2(e23.y)), h23, mul2(make_float2(bv.z, bv.w), gg));
+        h[j] = make_float4(h01.x, h01.y, h23.x, h23.y);
+        const float2 acc = fma2(make_float2(cv.z, cv.w), h23, mul2(make_float2(cv.x, cv.y), h01));
+        part[j] = acc.x + acc.y;
     }
-}
+    const float ysum = reduce_slots(part, q);
 
-// ---------------------------------------------------------------------------
-// mb_scan_verify: from h0, scan k drafted bytes; write every state to h_all.
-template <typename T>
-__global__ void __launch_bounds__(kThreads) verify_kernel(ScanParams p) {
-    const int q = threadIdx.x & 3;
-    const int64_t nchan = p.batch * p.d_inner;
-    const int64_t ch = (int64_t)blockIdx.x * kChanPerCta + (threadIdx.x >> 2);
-    const bool ok = ch < nchan;
-    const int64_t b = ok ? ch / p.d_inner : 0;
-    const int64_t d = ok ? ch - b * p.d_inner : 0;
-    const int64_t L = p.seqlen, D = p.d_inner;
-    const T *x = static_cast<const T *>(p.x);
-    const T *z = static_cast<const T *>(p.z);
-    const T *dt = static_cast<const T *>(p.dt);
-    const T *Bm = static_cast<const T *>(p.B);
-    const T *Cm = static_cast<const T *>(p.C);
-    T *y = static_cast<T *>(p.y);
-
-    float4 h = (ok && p.h0) ? __ldg(reinterpret_cast<const float4 *>(p.h0 + ch * kDState) + q)
-                            : make_float4(0.f, 0.f, 0.f, 0.f);
-    float4 a2 = ldg4(p.A + d * kDState + 4 * q);
-    a2.x *= kLog2e; a2.y *= kLog2e; a2.z *= kLog2e; a2.w *= kLog2e;
-    const float bias = p.dt_bias ? __ldg(p.dt_bias + d) : 0.f;
-    const float Dd = p.D ? __ldg(p.D + d) : 0.f;
-
-#pragma unroll 4
-    for (int64_t t = 0; t < L; ++t) {
-        const int64_t i = (b * L + t) * D + d;
-        const float xv = ldg1(x + i);
-        const float delta = softplus(ldg1(dt + i) + bias);
-        const float4 bv = ldg4(Bm + (b * L + t) * kDState + 4 * q);
-        const float4 cv = ldg4(Cm + (b * L + t) * kDState + 4 * q);
-        float part = lane_update(h, a2, delta, delta * xv, bv, cv);
-        part += __shfl_xor_sync(kFull, part, 1);
-        part += __shfl_xor_sync(kFull, part, 2);
-        if (ok) {
-            __stcs(reinterpret_cast<float4 *>(p.h_out + ((b * L + t) * D + d) * kDState) + q, h);
-            if (q == 0) {
-                float out = part + Dd * xv;
-                if (z) out *= silu(ldg1(z + i));
-                y[i] = from_f32<T>(out);
-            }
-        }
+#pragma unroll
+    for (int j = 0; j < kSlots; ++j) {
+        const int64_t ch = wbase + 8 * j + g;
+        if (ch < nchan) __stcs(state + ch * (kDState / 4) + q, h[j]);
     }
+    if (mok) static_cast<T *>(p.y)[mc] = from_f32<T>((ysum + xd) * sz);
 }
 
 // ---------------------------------------------------------------------------
 // mb_rollback: h_out[s] = accept[s] == 0 ? h0[s] : h_all[s, accept[s] - 1].
-__global__ void __launch_bounds__(kThreads)
-rollback_kernel(const float4 *__restrict__ h0, const float4 *__restrict__ h_all,
+// Each thread copies kRbVec float4s of one stream (per_stream is a multiple of
+// 4 float4s since d_inner * 16 floats = 4 * d_inner float4s).
+constexpr int kRbThreads = 256;
+constexpr int kRbVec = 4;
+
+__global__ void __launch_bounds__(kRbThreads)
+rollback_kernel(const float4 *h0 /* may alias h_out */, const float4 *__restrict__ h_all,
                 const int32_t *__restrict__ accept, float4 *h_out, int64_t batch, int64_t k,
                 int64_t per_stream /* float4s */, StatusBlock *status) {
-    const int64_t total = batch * per_stream;
-    for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < total;
-         i += (int64_t)gridDim.x * kThreads) {
-        const int64_t s = i / per_stream;
-        const int64_t j = i - s * per_stream;
-        const int a = __ldg(accept + s);
-        if (a < 0 || a > k) {
-            if (j == 0) report(status, 1 /* MB_ERR_INVALID_ARG */, s);
-            continue;
-        }
-        float4 v;
-        if (a == 0)
-            v = h0 ? __ldg(h0 + i) : make_float4(0.f, 0.f, 0.f, 0.f);
-        else
-            v = __ldcs(h_all + (s * k + (a - 1)) * per_stream + j);
-        h_out[i] = v;
+    const int64_t i0 = ((int64_t)blockIdx.x * kRbThreads + threadIdx.x) * kRbVec;
+    if (i0 >= batch * per_stream) return;
+    const int64_t s = i0 / per_stream;
+    const int64_t j0 = i0 - s * per_stream;
+    const int a = __ldg(accept + s);
+    if (a < 0 || a > k) {
+        if (j0 == 0) report(status, 1 /* MB_ERR_INVALID_ARG */, s);
+        return;
     }
+    float4 v[kRbVec];
+    const float4 *src = a == 0 ? (h0 ? h0 + i0 : nullptr) : h_all + (s * k + (a - 1)) * per_stream + j0;
+#pragma unroll
+    for (int u = 0; u < kRbVec; ++u) v[u] = src ? __ldcs(src + u) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int u = 0; u < kRbVec; ++u) h_out[i0 + u] = v[u];
 }
 
 }  // namespace
 
 cudaError_t launch_step(const ScanParams &p, bool bf16, cudaStream_t s) {
-    constexpr int CPT = 2;
     const int64_t nchan = p.batch * p.d_inner;
-    const int64_t grid = (nchan + kChanPerCta * CPT - 1) / (kChanPerCta * CPT);
+    const int64_t grid = (nchan + kStepChPerCta - 1) / kStepChPerCta;
     if (grid == 0) return cudaSuccess;
     if (bf16)
-        step_kernel<__nv_bfloat16, CPT><<<(unsigned)grid, kThreads, 0, s>>>(p);
+        step_kernel<__nv_bfloat16><<<(unsigned)grid, kStepThreads, 0, s>>>(p);
     else
-        step_kernel<float, CPT><<<(unsigned)grid, kThreads, 0, s>>>(p);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s) {
-    const int64_t nchan = p.batch * p.d_inner;
-    const int64_t grid = (nchan + kChanPerCta - 1) / kChanPerCta;
-    if (grid == 0 || p.seqlen == 0) return cudaSuccess;
-    if (bf16)
-        verify_kernel<__nv_bfloat16><<<(unsigned)grid, kThreads, 0, s>>>(p);
-    else
-        verify_kernel<float><<<(unsigned)grid, kThreads, 0, s>>>(p);
+        step_kernel<float><<<(unsigned)grid, kStepThreads, 0, s>>>(p);
     return cudaGetLastError();
 }
 
@@ -178,11 +148,10 @@ cudaError_t launch_rollback(const float *h0, const float *h_all, const int32_t *
                             float *h_out, int64_t batch, int64_t k, int64_t d_inner,
                             StatusBlock *status, cudaStream_t s) {
     const int64_t per = d_inner * kDState / 4;
-    const int64_t total = batch * per;
-    if (total == 0) return cudaSuccess;
-    int64_t grid = (total + kThreads - 1) / kThreads;
-    if (grid > 152 * 16) grid = 152 * 16;
-    rollback_kernel<<<(unsigned)grid, kThreads, 0, s>>>(
+    const int64_t threads = batch * per / kRbVec;
+    if (threads == 0) return cudaSuccess;
+    const int64_t grid = (threads + kRbThreads - 1) / kRbThreads;
+    rollback_kernel<<<(unsigned)grid, kRbThreads, 0, s>>>(
         reinterpret_cast<const float4 *>(h0), reinterpret_cast<const float4 *>(h_all), accept,
         reinterpret_cast<float4 *>(h_out), batch, k, per, status);
     return cudaGetLastError();

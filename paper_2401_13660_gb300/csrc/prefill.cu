@@ -1,191 +1,438 @@
 // Prefill scan of the selective-scan layer core (MambaByte Section 2,
-// "Implementation: parallel scans"; Eq. 2-3; Table 6 output and gating).
+// "Implementation: parallel scans"; Eq. 2-3; Table 6 output and gating), and
+// the speculative-decoding verify scan (Algorithm 1), which is the same scan
+// that also streams every per-position state to h_all.
 //
 // Work decomposition. Every (batch row, channel) pair is an independent
-// linear recurrence over L steps with a 16-float state, so the kernel is
-// channel-parallel and runs each channel's recurrence sequentially in time
-// (the cheapest evaluation order in operations: one FMA per state per step;
-// a time-parallel scan with the associative operator of Section 2 would add
-// work per element). A CTA owns kCh channels of one batch row; four lanes per
-// channel each hold 4 of the 16 states in registers (fp32) for the whole
-// sequence.
+// linear recurrence over L steps with a 16-float state (A is diagonal, so the
+// scan of Section 2 is element-wise). The kernel is channel-parallel and runs
+// each channel's recurrence sequentially in time, the evaluation order with
+// the fewest operations (one Abar, one FMA for h and one FMA for C.h per state
+// and step); the associative operator of Section 2 is only needed to split a
+// span, which the h0 / h_last interface does across calls.
 //
-// Per chunk of kT time steps the CTA
-//   1. loads the raw dt, x, z [kT, kCh] and B, C [kT, 16] tiles (coalesced,
-//      issued one chunk ahead into registers so the loads overlap the scan),
-//   2. converts them once per (t, channel) into shared memory:
-//      (Delta, Delta*x) with Delta = softplus(dt + bias), D*x, z, and B, C as
-//      fp32 (so the softplus is paid once per channel-byte, not per lane),
-//   3. scans: per step and state, Abar = 2^(Delta * A*log2 e) on the SFU and
-//      h = Abar*h + B*(Delta*x); each lane writes its share of C.h,
-//   4. reduces the four shares per (t, channel), adds D*x, applies silu(z)
-//      and stores y (32 consecutive channels per warp store).
-// Steps past L are padded with Delta = 0, which leaves the state unchanged.
+// A CTA (4 warps) owns CH = 128 / LPC channels of one batch row for the whole
+// span. LPC lanes share a channel, each keeping 16 / LPC of its fp32 states in
+// registers. The state index varies slowest across a warp, so the 8 lanes of
+// each quarter-warp read the same B, C values (a shared-memory broadcast).
+//
+// Pipeline, per chunk of kT = 16 time steps:
+//  * one thread keeps a STAGES-deep ring of 3-D TMA tile loads in flight:
+//    dt, x, z [kT x CH] and B, C [kT x 16], one mbarrier per stage (bounded
+//    waits, tma.cuh);
+//  * the CTA converts a chunk once per (t, channel) into fp32 in shared
+//    memory: (Delta, Delta*x) with Delta = softplus(dt + bias), (D*x,
+//    silu(z)), and B, C;
+//  * each lane scans the chunk: Abar = 2^(Delta * A*log2 e) on the SFU for all
+//    kT steps, then h = Abar*h + B*(Delta*x) and its share of C.h in packed
+//    f32x2 arithmetic; groups of LPC steps are reduced across the LPC lanes
+//    of a channel with log2(LPC) shuffle rounds, each lane finishing one
+//    output y = (C.h + D*x) * silu(z), which goes to a shared-memory tile that
+//    one thread writes out with a TMA store.
+//  Loop iteration i converts chunk i+1 and scans chunk i in one basic block,
+//  so every warp has two independent instruction streams to interleave; one
+//  CTA barrier per chunk orders them.
+// Steps at or beyond L are converted with Delta = 0, which leaves h unchanged.
+#include <string.h>
+
 #include "common.cuh"
+#include "tma.cuh"
 
 namespace mbscan {
 namespace {
 
-constexpr int kCh = 32;              // channels per CTA
-constexpr int kT = 16;               // time steps per chunk
-constexpr int kThreads = kCh * 4;    // four lanes per channel
+constexpr int kT = 16;            // time steps per chunk
+constexpr int kThreads = 128;     // 4 warps
+#ifndef MB_PREFILL_LPC
+#define MB_PREFILL_LPC 4
+#endif
+constexpr int kPrefillLanesPerChannel = MB_PREFILL_LPC;
+constexpr int kPrefillStages = 4;  // TMA ring depth for long spans
+constexpr int kVerifyStages = 2;   // verify spans are short
 
+// Lane geometry: LPC lanes share one channel, each holding kSPL states.
+template <int LPC>
+struct Geom {
+    static constexpr int kSPL = kDState / LPC;     // states per lane
+    static constexpr int kPairs = kSPL / 2;        // float2 state pairs per lane
+    static constexpr int kChPerWarp = 32 / LPC;
+    static constexpr int kCh = 4 * kChPerWarp;     // channels per CTA
+};
+
+template <typename T, int CH>
+struct Raw {  // TMA destinations; every member offset is a multiple of 128 B
+    T dt[kT][CH];
+    T x[kT][CH];
+    T z[kT][CH];
+    T B[kT][kDState];
+    T C[kT][kDState];
+};
+
+template <int CH>
+struct Conv {
+    float2 dg[kT][CH];          // (Delta, Delta*x)
+    float2 xs[kT][CH];          // (D*x, silu(z)); silu(z) = 1 without a gate
+    float bc[kT][2 * kDState];  // B[0..15], C[0..15]
+};
+
+template <typename T, int CH, int STAGES>
 struct Smem {
-    float2 dd[2][kT][kCh];   // (Delta, Delta*x)
-    float bm[2][kT][kDState];
-    float cm[2][kT][kDState];
-    float zg[2][kT][kCh];    // gate input z
-    float xd[2][kT][kCh];    // D*x
-    float part[kT][kCh * 4]; // per-lane shares of C.h
+    Raw<T, CH> raw[STAGES];
+    Conv<CH> cv[2];
+    T ys[2][kT][CH];            // output tiles, written out by TMA stores
+    uint64_t full[STAGES];
 };
 
-// Raw chunk held in registers between the global load and the conversion.
-struct Raw {
-    float4 dt, x, z;   // 4 consecutive channels at one time step
-    float2 b, c;       // 2 consecutive states at one time step
+struct PrefillArgs {
+    CUtensorMap tm_dt, tm_x, tm_z, tm_B, tm_C, tm_y;
+    ScanParams p;
+    int has_gate;
 };
 
-template <typename T>
-__device__ __forceinline__ Raw load_chunk(const ScanParams &p, int64_t b, int64_t d0, int64_t t0) {
-    const int tid = threadIdx.x;
-    const int t = tid >> 3;               // 0..15
-    const int c4 = (tid & 7) * 4;         // 0..28
-    const int64_t tt = t0 + t;
-    Raw r;
-    const float4 zero4 = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (tt < p.seqlen && d0 + c4 < p.d_inner) {
-        const int64_t i = (b * p.seqlen + tt) * p.d_inner + d0 + c4;
-        r.dt = ldg4(static_cast<const T *>(p.dt) + i);
-        r.x = ldg4(static_cast<const T *>(p.x) + i);
-        r.z = p.z ? ldg4(static_cast<const T *>(p.z) + i) : zero4;
-    } else {
-        r.dt = zero4; r.x = zero4; r.z = zero4;
-    }
-    const int n2 = (tid & 7) * 2;
-    if (tt < p.seqlen) {
-        const int64_t j = (b * p.seqlen + tt) * kDState + n2;
-        r.b = ldg2(static_cast<const T *>(p.B) + j);
-        r.c = ldg2(static_cast<const T *>(p.C) + j);
-    } else {
-        r.b = make_float2(0.f, 0.f); r.c = make_float2(0.f, 0.f);
-    }
-    return r;
+template <typename T, int CH, int STAGES>
+__device__ __forceinline__ void issue_chunk(Smem<T, CH, STAGES> &s, const PrefillArgs &a, int stage,
+                                            int64_t chunk, int d0, int b) {
+    constexpr uint32_t tok = kT * CH * sizeof(T), bc = kT * kDState * sizeof(T);
+    const uint32_t bytes = (a.has_gate ? 3 : 2) * tok + 2 * bc;
+    uint64_t *bar = &s.full[stage];
+    mbar_arrive_expect_tx(bar, bytes);
+    const int t = (int)(chunk * kT);
+    Raw<T, CH> &r = s.raw[stage];
+    tma_load_3d(&r.dt[0][0], &a.tm_dt, bar, d0, t, b);
+    tma_load_3d(&r.x[0][0], &a.tm_x, bar, d0, t, b);
+    if (a.has_gate) tma_load_3d(&r.z[0][0], &a.tm_z, bar, d0, t, b);
+    tma_load_3d(&r.B[0][0], &a.tm_B, bar, 0, t, b);
+    tma_load_3d(&r.C[0][0], &a.tm_C, bar, 0, t, b);
 }
 
-__device__ __forceinline__ void convert_store(Smem &s, int buf, const Raw &r, int64_t b,
-                                              int64_t d0, int64_t t0, const ScanParams &p) {
-    const int tid = threadIdx.x;
-    const int t = tid >> 3;
-    const int c4 = (tid & 7) * 4;
-    const bool valid = (t0 + t < p.seqlen) && (d0 + c4 < p.d_inner);
-    const float dtv[4] = {r.dt.x, r.dt.y, r.dt.z, r.dt.w};
-    const float xv[4] = {r.x.x, r.x.y, r.x.z, r.x.w};
-    const float zv[4] = {r.z.x, r.z.y, r.z.z, r.z.w};
+// Two adjacent channels of the input dtype, widened to fp32.
+__device__ __forceinline__ float2 ld_pair(const float *p) { return *reinterpret_cast<const float2 *>(p); }
+__device__ __forceinline__ float2 ld_pair(const __nv_bfloat16 *p) {
+    const unsigned u = *reinterpret_cast<const unsigned *>(p);
+    return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
+}
+
+// Per-thread constants of the conversion role: thread converts the adjacent
+// channel pair (2 cp, 2 cp + 1) at steps th, th + kRows, ...
+template <int CH>
+struct ConvRole {
+    static constexpr int kPairsPerRow = CH / 2;
+    static constexpr int kRows = kThreads / kPairsPerRow;   // step rows per pass
+    static constexpr int kPasses = kT / kRows;
+    int cp, th;
+    float2 bias, dsk;
+    bool ok;
+};
+
+// Convert one chunk: raw TMA tiles -> fp32 (Delta, Delta*x), (D*x, silu z), B, C.
+template <typename T, int CH>
+__device__ __forceinline__ void convert(Conv<CH> &cv, const Raw<T, CH> &r, const ConvRole<CH> &cr,
+                                        int64_t t0, int64_t L, bool gate) {
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        float delta = 0.f, dx = 0.f, xdv = 0.f;
-        if (valid) {
-            const int64_t d = d0 + c4 + j;
-            delta = softplus(dtv[j] + (p.dt_bias ? __ldg(p.dt_bias + d) : 0.f));
-            dx = delta * xv[j];
-            xdv = (p.D ? __ldg(p.D + d) : 0.f) * xv[j];
+    for (int k = 0; k < ConvRole<CH>::kPasses; ++k) {
+        const int t = cr.th + ConvRole<CH>::kRows * k;
+        const int c = 2 * cr.cp;
+        float4 dg = make_float4(0.f, 0.f, 0.f, 0.f), xs = make_float4(0.f, 1.f, 0.f, 1.f);
+        if (cr.ok && t0 + t < L) {
+            const float2 xv = ld_pair(&r.x[t][c]);
+            const float2 dv = ld_pair(&r.dt[t][c]);
+            const float d0 = softplus(dv.x + cr.bias.x), d1 = softplus(dv.y + cr.bias.y);
+            dg = make_float4(d0, d0 * xv.x, d1, d1 * xv.y);
+            xs.x = cr.dsk.x * xv.x;
+            xs.z = cr.dsk.y * xv.y;
+            if (gate) {
+                const float2 zv = ld_pair(&r.z[t][c]);
+                xs.y = silu(zv.x);
+                xs.w = silu(zv.y);
+            }
         }
-        s.dd[buf][t][c4 + j] = make_float2(delta, dx);
-        s.xd[buf][t][c4 + j] = xdv;
-        s.zg[buf][t][c4 + j] = zv[j];
+        *reinterpret_cast<float4 *>(&cv.dg[t][c]) = dg;
+        *reinterpret_cast<float4 *>(&cv.xs[t][c]) = xs;
     }
-    const int n2 = (tid & 7) * 2;
-    s.bm[buf][t][n2] = r.b.x;
-    s.bm[buf][t][n2 + 1] = r.b.y;
-    s.cm[buf][t][n2] = r.c.x;
-    s.cm[buf][t][n2 + 1] = r.c.y;
+    {   // B, C: kT steps x 32 values, 4 per thread
+        const int t = threadIdx.x >> 3, k4 = (threadIdx.x & 7) * 4;
+        const T *src = k4 < kDState ? &r.B[t][k4] : &r.C[t][k4 - kDState];
+        const float2 lo = ld_pair(src), hi = ld_pair(src + 2);
+        *reinterpret_cast<float4 *>(&cv.bc[t][k4]) = make_float4(lo.x, lo.y, hi.x, hi.y);
+    }
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kThreads) prefill_kernel(ScanParams p) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    Smem &s = *reinterpret_cast<Smem *>(smem_raw);
-    const int tid = threadIdx.x;
-    const int64_t b = blockIdx.y;
-    const int64_t d0 = (int64_t)blockIdx.x * kCh;
-    const int c = tid >> 2;   // channel within the CTA (scan role)
-    const int q = tid & 3;    // state quarter
-    const int64_t d = d0 + c;
-    const bool chan_ok = d < p.d_inner;
-
-    float4 h = make_float4(0.f, 0.f, 0.f, 0.f);
-    float4 a2 = h;
-    if (chan_ok) {
-        if (p.h0) h = __ldg(reinterpret_cast<const float4 *>(p.h0 + (b * p.d_inner + d) * kDState) + q);
-        a2 = ldg4(p.A + d * kDState + 4 * q);
-        a2.x *= kLog2e; a2.y *= kLog2e; a2.z *= kLog2e; a2.w *= kLog2e;
+// Sum the LPC per-lane shares of C.h for LPC consecutive steps so that lane q
+// ends with the full sum of step q of the group (a transposed reduction:
+// log2(LPC) shuffle rounds per LPC steps instead of per step). The lanes of
+// one channel are 32 / LPC apart (q is the slowest-varying lane index).
+template <int LPC>
+__device__ __forceinline__ float reduce_steps(const float (&part)[LPC], int q) {
+    if constexpr (LPC == 2) {
+        const float keep = q ? part[1] : part[0];
+        const float send = q ? part[0] : part[1];
+        return keep + __shfl_xor_sync(kFull, send, 16);
+    } else {
+        static_assert(LPC == 4, "LPC must be 2 or 4");
+        const bool hi = (q & 2) != 0;
+        float k0 = hi ? part[2] : part[0], k1 = hi ? part[3] : part[1];
+        const float s0 = hi ? part[0] : part[2], s1 = hi ? part[1] : part[3];
+        k0 += __shfl_xor_sync(kFull, s0, 16);
+        k1 += __shfl_xor_sync(kFull, s1, 16);
+        const bool odd = (q & 1) != 0;
+        const float keep = odd ? k1 : k0, send = odd ? k0 : k1;
+        return keep + __shfl_xor_sync(kFull, send, 8);
     }
+}
 
-    const int64_t nchunks = (p.seqlen + kT - 1) / kT;
-    Raw r = load_chunk<T>(p, b, d0, 0);
-    convert_store(s, 0, r, b, d0, 0, p);
+template <typename T, int LPC, int STAGES, bool kStoreAll>
+__global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant__ PrefillArgs a) {
+    using G = Geom<LPC>;
+    constexpr int CH = G::kCh;
+    using S = Smem<T, CH, STAGES>;
+    extern __shared__ unsigned char smem_dyn[];
+    S &s = *reinterpret_cast<S *>((reinterpret_cast<uintptr_t>(smem_dyn) + 127) &
+                                  ~static_cast<uintptr_t>(127));
+    const ScanParams &p = a.p;
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    const int b = blockIdx.y;
+    const int d0 = blockIdx.x * CH;
+    const int64_t L = p.seqlen, D = p.d_inner;
+    const int64_t nchunks = (L + kT - 1) / kT;
+    const bool gate = a.has_gate != 0;
+
+    if (tid == 0) {
+        for (int st = 0; st < STAGES; ++st) mbar_init(&s.full[st], 1);
+        fence_mbar_init();
+    }
     __syncthreads();
+    if (tid == 0) {
+        for (int st = 0; st < STAGES && st < nchunks; ++st) issue_chunk(s, a, st, st, d0, b);
+    }
 
-    T *y = static_cast<T *>(p.y);
-    const bool gate = p.z != nullptr;
-    for (int64_t ci = 0; ci < nchunks; ++ci) {
-        const int buf = (int)(ci & 1);
-        const int64_t t0 = ci * kT;
-        if (ci + 1 < nchunks) r = load_chunk<T>(p, b, d0, t0 + kT);
+    // ---- conversion role
+    ConvRole<CH> cr;
+    cr.cp = tid % ConvRole<CH>::kPairsPerRow;
+    cr.th = tid / ConvRole<CH>::kPairsPerRow;
+    {
+        const int64_t dc = d0 + 2 * cr.cp;   // D % 8 == 0: both channels valid or neither
+        cr.ok = dc < D;
+        cr.bias = (cr.ok && p.dt_bias) ? __ldg(reinterpret_cast<const float2 *>(p.dt_bias + dc))
+                                       : make_float2(0.f, 0.f);
+        cr.dsk = (cr.ok && p.D) ? __ldg(reinterpret_cast<const float2 *>(p.D + dc)) : make_float2(0.f, 0.f);
+    }
 
-#pragma unroll 4
-        for (int t = 0; t < kT; ++t) {
-            const float2 dd = s.dd[buf][t][c];
-            const float4 bv = *reinterpret_cast<const float4 *>(&s.bm[buf][t][4 * q]);
-            const float4 cv = *reinterpret_cast<const float4 *>(&s.cm[buf][t][4 * q]);
-            h.x = fmaf(ex2(dd.x * a2.x), h.x, bv.x * dd.y);
-            h.y = fmaf(ex2(dd.x * a2.y), h.y, bv.y * dd.y);
-            h.z = fmaf(ex2(dd.x * a2.z), h.z, bv.z * dd.y);
-            h.w = fmaf(ex2(dd.x * a2.w), h.w, bv.w * dd.y);
-            s.part[t][tid] = fmaf(cv.x, h.x, fmaf(cv.y, h.y, fmaf(cv.z, h.z, cv.w * h.w)));
-        }
-        __syncthreads();
-
-        // Epilogue: warp w handles time steps w, w+4, ...; lane = channel.
-        {
-            const int ec = tid & 31;
-            const int64_t ed = d0 + ec;
+    // ---- scan role: channel c, states kSPL*q .. kSPL*q + kSPL-1
+    const int c = warp * G::kChPerWarp + lane % G::kChPerWarp;
+    const int q = lane / G::kChPerWarp;
+    const int64_t d = d0 + c;
+    const bool chan_ok = d < D;
+    float2 h[G::kPairs], a2[G::kPairs];
 #pragma unroll
-            for (int t = tid >> 5; t < kT; t += 4) {
-                if (t0 + t < p.seqlen && ed < p.d_inner) {
-                    const float4 pp = *reinterpret_cast<const float4 *>(&s.part[t][ec * 4]);
-                    float out = (pp.x + pp.y) + (pp.z + pp.w) + s.xd[buf][t][ec];
-                    if (gate) out *= silu(s.zg[buf][t][ec]);
-                    y[(b * p.seqlen + t0 + t) * p.d_inner + ed] = from_f32<T>(out);
+    for (int k = 0; k < G::kPairs; ++k) { h[k] = make_float2(0.f, 0.f); a2[k] = h[k]; }
+    if (chan_ok) {
+        const float2 *Ap = reinterpret_cast<const float2 *>(p.A + d * kDState + G::kSPL * q);
+        const float2 *hp = reinterpret_cast<const float2 *>(p.h0 + ((int64_t)b * D + d) * kDState + G::kSPL * q);
+#pragma unroll
+        for (int k = 0; k < G::kPairs; ++k) {
+            const float2 av = __ldg(Ap + k);
+            a2[k] = make_float2(av.x * kLog2e, av.y * kLog2e);
+            if (p.h0) h[k] = __ldg(hp + k);
+        }
+    }
+
+    // ---- prologue: chunk 0
+    bool ok = nchunks > 0 ? mbar_wait(&s.full[0], 0) : true;
+    if (ok && nchunks > 0) convert(s.cv[0], s.raw[0], cr, 0, L, gate);
+    if (__syncthreads_or(ok ? 0 : 1)) {
+        if (tid == 0) {
+            report(p.status, 4 /* MB_ERR_TIMEOUT */, 0);
+            for (int j = 0; j < STAGES && j < nchunks; ++j) mbar_wait(&s.full[j], 0);
+        }
+        return;
+    }
+    if (tid == 0 && STAGES < nchunks) {
+        fence_proxy_async_smem();
+        issue_chunk(s, a, 0, STAGES, d0, b);
+    }
+
+    for (int64_t i = 0; i < nchunks; ++i) {
+        const int64_t t0 = i * kT;
+        const bool has_next = i + 1 < nchunks;
+        // (1) chunk i+1: wait for its tiles and convert them
+        const int nst = (int)((i + 1) % STAGES);
+        ok = has_next ? mbar_wait(&s.full[nst], (uint32_t)(((i + 1) / STAGES) & 1)) : true;
+        if (has_next && ok) convert(s.cv[(i + 1) & 1], s.raw[nst], cr, t0 + kT, L, gate);
+
+        // (2) chunk i: decays of all kT steps, recurrence, shares of C.h
+        const Conv<CH> &cv = s.cv[i & 1];
+        float2 ab[kT][G::kPairs];
+        float gx[kT];
+#pragma unroll
+        for (int t = 0; t < kT; ++t) {
+            const float2 dg = cv.dg[t][c];
+            const float2 dd = make_float2(dg.x, dg.x);
+            gx[t] = dg.y;
+#pragma unroll
+            for (int k = 0; k < G::kPairs; ++k) {
+                const float2 e = mul2(dd, a2[k]);
+                ab[t][k] = make_float2(ex2(e.x), ex2(e.y));
+            }
+        }
+        float part[kT];
+#pragma unroll
+        for (int t = 0; t < kT; ++t) {
+            const float2 gg = make_float2(gx[t], gx[t]);
+            float2 bp[G::kPairs], cp[G::kPairs];
+#pragma unroll
+            for (int k = 0; k < G::kPairs; k += 2) {
+                const float4 b4 = *reinterpret_cast<const float4 *>(&cv.bc[t][G::kSPL * q + 2 * k]);
+                const float4 c4 = *reinterpret_cast<const float4 *>(&cv.bc[t][kDState + G::kSPL * q + 2 * k]);
+                bp[k] = make_float2(b4.x, b4.y); bp[k + 1] = make_float2(b4.z, b4.w);
+                cp[k] = make_float2(c4.x, c4.y); cp[k + 1] = make_float2(c4.z, c4.w);
+            }
+            float2 acc[2];
+#pragma unroll
+            for (int k = 0; k < G::kPairs; ++k) {
+                h[k] = fma2(ab[t][k], h[k], mul2(bp[k], gg));
+                acc[k & 1] = k < 2 ? mul2(cp[k], h[k]) : fma2(cp[k], h[k], acc[k & 1]);
+            }
+            const float2 sum = add2(acc[0], acc[1]);
+            part[t] = sum.x + sum.y;
+            if constexpr (kStoreAll) {
+                if (chan_ok && t0 + t < L) {
+                    float2 *dst = reinterpret_cast<float2 *>(
+                        p.h_out + (((int64_t)b * L + t0 + t) * D + d) * kDState + G::kSPL * q);
+#pragma unroll
+                    for (int k = 0; k < G::kPairs; k += 2)
+                        __stcs(reinterpret_cast<float4 *>(dst + k),
+                               make_float4(h[k].x, h[k].y, h[k + 1].x, h[k + 1].y));
                 }
             }
         }
-        if (ci + 1 < nchunks) convert_store(s, buf ^ 1, r, b, d0, t0 + kT, p);
-        __syncthreads();
+        // (3) chunk i: reduce across the lanes of each channel, gate, stage y
+        T(&ys)[kT][CH] = s.ys[i & 1];
+#pragma unroll
+        for (int m = 0; m < kT / LPC; ++m) {
+            float grp[LPC];
+#pragma unroll
+            for (int u = 0; u < LPC; ++u) grp[u] = part[LPC * m + u];
+            const float ysum = reduce_steps<LPC>(grp, q);
+            const int t = LPC * m + q;
+            const float2 xs = cv.xs[t][c];
+            ys[t][c] = from_f32<T>((ysum + xs.x) * xs.y);
+        }
+        fence_proxy_async_smem();   // y tile -> visible to the TMA store below
+        if (tid == 0) bulk_wait_read_all();   // the store of chunk i-1 no longer reads its tile
+        if (__syncthreads_or(ok ? 0 : 1)) {
+            if (tid == 0) {
+                report(p.status, 4 /* MB_ERR_TIMEOUT */, i + 1);
+                for (int64_t j = i + 1; j < i + 1 + STAGES && j < nchunks; ++j)
+                    mbar_wait(&s.full[j % STAGES], (uint32_t)((j / STAGES) & 1));
+                bulk_wait_all();
+            }
+            return;
+        }
+        if (tid == 0) {
+            tma_store_3d(&a.tm_y, &ys[0][0], d0, (int)t0, b);
+            bulk_commit();
+            if (has_next && i + 1 + STAGES < nchunks) {
+                fence_proxy_async_smem();
+                issue_chunk(s, a, nst, i + 1 + STAGES, d0, b);
+            }
+        }
     }
+    if (tid == 0) bulk_wait_all();
 
-    if (p.h_out && chan_ok)
-        reinterpret_cast<float4 *>(p.h_out + (b * p.d_inner + d) * kDState)[q] = h;
+    if (!kStoreAll && p.h_out && chan_ok) {
+        float2 *hp = reinterpret_cast<float2 *>(p.h_out + ((int64_t)b * D + d) * kDState + G::kSPL * q);
+#pragma unroll
+        for (int k = 0; k < G::kPairs; ++k) hp[k] = h[k];
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Host side: tensor maps (encoded per call through the driver entry point, so
+// the library does not link libcuda) and the launch.
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                             &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            f = nullptr;
+        return reinterpret_cast<EncodeTiledFn>(f);
+    }();
+    return fn;
+}
+
+// [batch, L, inner] tensor with a (box_inner x kT x 1) box.
+bool make_map(CUtensorMap *m, const void *base, bool bf16, int64_t batch, int64_t L, int64_t inner,
+              int box_inner) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    const int64_t es = bf16 ? 2 : 4;
+    cuuint64_t dims[3] = {(cuuint64_t)inner, (cuuint64_t)L, (cuuint64_t)batch};
+    cuuint64_t strides[2] = {(cuuint64_t)(inner * es), (cuuint64_t)(L * inner * es)};
+    cuuint32_t box[3] = {(cuuint32_t)box_inner, (cuuint32_t)kT, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3,
+                     const_cast<void *>(base), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <typename T, int LPC, int STAGES, bool kStoreAll>
+cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
+    constexpr int kCh = Geom<LPC>::kCh;
+    const bool bf16 = sizeof(T) == 2;
+    PrefillArgs a;
+    memset(&a, 0, sizeof(a));
+    a.p = p;
+    a.has_gate = p.z != nullptr;
+    if (!make_map(&a.tm_dt, p.dt, bf16, p.batch, p.seqlen, p.d_inner, kCh) ||
+        !make_map(&a.tm_x, p.x, bf16, p.batch, p.seqlen, p.d_inner, kCh) ||
+        (p.z && !make_map(&a.tm_z, p.z, bf16, p.batch, p.seqlen, p.d_inner, kCh)) ||
+        !make_map(&a.tm_B, p.B, bf16, p.batch, p.seqlen, kDState, kDState) ||
+        !make_map(&a.tm_C, p.C, bf16, p.batch, p.seqlen, kDState, kDState) ||
+        !make_map(&a.tm_y, p.y, bf16, p.batch, p.seqlen, p.d_inner, kCh))
+        return cudaErrorInvalidValue;
+    const size_t smem = sizeof(Smem<T, kCh, STAGES>) + 128;
+    auto k = prefill_kernel<T, LPC, STAGES, kStoreAll>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const dim3 grid((unsigned)((p.d_inner + kCh - 1) / kCh), (unsigned)p.batch);
+    k<<<grid, kThreads, smem, s>>>(a);
+    return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s) {
-    if (p.batch == 0) return cudaSuccess;
-    const dim3 grid((unsigned)((p.d_inner + kCh - 1) / kCh), (unsigned)p.batch);
-    const size_t smem = sizeof(Smem);
-    if (bf16) {
-        auto k = prefill_kernel<__nv_bfloat16>;
-        cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        k<<<grid, kThreads, smem, s>>>(p);
-    } else {
-        auto k = prefill_kernel<float>;
-        cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        k<<<grid, kThreads, smem, s>>>(p);
+    if (p.batch == 0 || p.d_inner == 0) return cudaSuccess;
+    if (p.seqlen == 0) {
+        // Nothing to scan: the final state is the initial state.
+        if (!p.h_out) return cudaSuccess;
+        const size_t bytes = (size_t)p.batch * p.d_inner * kDState * sizeof(float);
+        if (p.h0) {
+            if (p.h0 == p.h_out) return cudaSuccess;
+            return cudaMemcpyAsync(p.h_out, p.h0, bytes, cudaMemcpyDeviceToDevice, s);
+        }
+        return cudaMemsetAsync(p.h_out, 0, bytes, s);
     }
-    return cudaGetLastError();
+    constexpr int LPC = kPrefillLanesPerChannel;
+    return bf16 ? launch_typed<__nv_bfloat16, LPC, kPrefillStages, false>(p, s)
+                : launch_typed<float, LPC, kPrefillStages, false>(p, s);
+}
+
+cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s) {
+    if (p.batch == 0 || p.d_inner == 0 || p.seqlen == 0) return cudaSuccess;
+    constexpr int LPC = kPrefillLanesPerChannel;
+    return bf16 ? launch_typed<__nv_bfloat16, LPC, kVerifyStages, true>(p, s)
+                : launch_typed<float, LPC, kVerifyStages, true>(p, s);
 }
 
 }  // namespace mbscan

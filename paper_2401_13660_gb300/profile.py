@@ -1,0 +1,109 @@
+"""Launch one entry point on a named workload, for profilers and quick timing.
+
+    python -m paper_2401_13660_gb300.profile --entry prefill \
+        --workload mambabyte353m_prefill_b8_L8192 --iters 5
+
+Inputs are drawn on the GPU with the seeded generator of `inputs`; each
+iteration launches the entry point once through the C ABI on one stream.
+Prints the mean device time per launch (CUDA events) and the algorithmic-byte
+rate. For the decode step, `--layers` distinct state/input sets are cycled so
+that the working set exceeds the 129 MB L2 (default 4 layers, 643 MB).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+import torch
+
+from . import mbscan as mb
+from .inputs import WORKLOADS, workload_inputs
+
+N_STATE = 16
+
+
+def algorithmic_bytes(entry: str, w, s_in: int) -> int:
+    b, L, D, N = w.batch, w.seqlen, w.d_inner, N_STATE
+    params = D * N * 4 + 2 * D * 4
+    if entry in ("prefill", "verify"):
+        rd = 3 * b * L * D * s_in + 2 * b * L * N * s_in + params
+        rd += b * D * N * 4 if (w.h0 != "zeros" or entry == "verify") else 0
+        wr = b * L * D * s_in + (b * D * N * 4 if entry == "prefill" else b * L * D * N * 4)
+        return rd + wr
+    if entry == "rollback":
+        return 2 * b * D * N * 4 + b * 4
+    if entry == "step":
+        return 2 * b * D * N * 4 + 3 * b * D * s_in + 2 * b * N * s_in + params + b * D * s_in
+    raise ValueError(entry)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--entry", choices=["prefill", "verify", "rollback", "step"], required=True)
+    ap.add_argument("--workload", required=True, choices=sorted(WORKLOADS))
+    ap.add_argument("--iters", type=int, default=5)
+    ap.add_argument("--layers", type=int, default=4, help="state sets cycled by --entry step")
+    a = ap.parse_args()
+    w = WORKLOADS[a.workload]
+    dev = torch.device("cuda:0")
+    mb.load_library()
+    nsets = a.layers if a.entry == "step" else 1
+    sets = []
+    for layer in range(nsets):
+        inp = workload_inputs(w, dev, layer=layer)
+        x = inp["x"]
+        inp["y"] = torch.empty_like(x)
+        inp["ws"] = torch.zeros(256, dtype=torch.uint8, device=dev)
+        if inp["h0"] is None and a.entry in ("verify", "rollback", "step"):
+            inp["h0"] = torch.zeros(w.batch, w.d_inner, N_STATE, device=dev)
+        if a.entry == "prefill":
+            inp["h_last"] = torch.empty(w.batch, w.d_inner, N_STATE, device=dev)
+        if a.entry in ("verify", "rollback"):
+            inp["h_all"] = torch.empty(w.batch, w.seqlen, w.d_inner, N_STATE, device=dev)
+            inp["h_out"] = torch.empty_like(inp["h0"])
+            if "accept" not in inp:
+                inp["accept"] = torch.randint(0, w.seqlen + 1, (w.batch,), device=dev,
+                                              dtype=torch.int32)
+        if a.entry == "step":
+            for k in ("x", "z", "dt", "B", "C", "y"):
+                inp[k] = inp[k][:, :1].contiguous()
+            inp["state"] = inp["h0"].clone()
+        sets.append(inp)
+    if a.entry == "rollback":
+        s0 = sets[0]
+        mb.mb_scan_verify(s0["x"], s0["dt"], s0["B"], s0["C"], s0["A"], s0["y"], s0["h_all"],
+                          z=s0["z"], D=s0["D"], dt_bias=s0["dt_bias"], h0=s0["h0"], ws=s0["ws"])
+
+    stream = torch.cuda.Stream(dev)
+
+    def launch(s):
+        if a.entry == "prefill":
+            mb.mb_scan_prefill(s["x"], s["dt"], s["B"], s["C"], s["A"], s["y"], z=s["z"], D=s["D"],
+                               dt_bias=s["dt_bias"], h0=s["h0"], h_last=s["h_last"], ws=s["ws"],
+                               stream=stream)
+        elif a.entry == "verify":
+            mb.mb_scan_verify(s["x"], s["dt"], s["B"], s["C"], s["A"], s["y"], s["h_all"], z=s["z"],
+                              D=s["D"], dt_bias=s["dt_bias"], h0=s["h0"], ws=s["ws"], stream=stream)
+        elif a.entry == "rollback":
+            mb.mb_rollback(s["h0"], s["h_all"], s["accept"], s["h_out"], ws=s["ws"], stream=stream)
+        else:
+            mb.mb_step(s["x"], s["dt"], s["B"], s["C"], s["A"], s["y"], s["state"], z=s["z"],
+                       D=s["D"], dt_bias=s["dt_bias"], stream=stream)
+
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    with torch.cuda.stream(stream):
+        launch(sets[0])
+        ev[0].record(stream)
+        for i in range(a.iters):
+            launch(sets[i % nsets])
+        ev[1].record(stream)
+    stream.synchronize()
+    us = 1e3 * ev[0].elapsed_time(ev[1]) / max(a.iters, 1)
+    nbytes = algorithmic_bytes(a.entry, w, 2 if w.dtype == "bf16" else 4)
+    print(json.dumps({"entry": a.entry, "workload": w.name, "iters": a.iters, "us_per_launch": round(us, 3),
+                      "algorithmic_bytes": nbytes, "GB/s": round(nbytes / (us * 1e-6) / 1e9, 1)}))
+
+
+if __name__ == "__main__":
+    main()
