@@ -6,22 +6,50 @@
 // Both are HBM-streaming kernels. A (batch row, channel) pair owns 16 fp32
 // states (64 contiguous bytes). In the step kernel four lanes share a channel,
 // each holding 4 states in one float4, so a warp moves 512 contiguous bytes
-// of state per instruction; each lane group serves kSlots channels so that
-// every lane has kSlots independent 16-byte state loads in flight.
+// of state per instruction.
 #include "common.cuh"
+#include <string.h>
+
 #include "tma.cuh"
 
 namespace mbscan {
 namespace {
 
-constexpr int kStepThreads = 256;
-constexpr int kSlots = 4;                                       // channels per lane group
-constexpr int kStepChPerWarp = 8 * kSlots;                      // 32
-constexpr int kStepChPerCta = kStepChPerWarp * (kStepThreads / 32);  // 256
+constexpr int kStepConsumers = 8;                          // consumer warps
+constexpr int kStepThreads = 32 * (kStepConsumers + 1);    // + one producer warp
+constexpr int kStepCh = 8 * kStepConsumers;                // 64 channels per tile
+constexpr int kStepRows = 4;                               // batch rows per tile
+constexpr int kStepStages = 4;
 
-// Lane q of a 4-lane group holds the group's shares part[0..3] (one per
-// slot); return the full 4-lane sum of slot q (two shuffle rounds).
-__device__ __forceinline__ float reduce_slots(const float (&part)[4], int q) {
+// One tile of the decode step in shared memory (TMA destinations; every member
+// offset is a multiple of 128 bytes for both dtypes).
+template <typename T>
+struct StepStage {
+    float state[kStepRows][kStepCh][kDState];   // 16 KB
+    T x[kStepRows][kStepCh];
+    T dt[kStepRows][kStepCh];
+    T z[kStepRows][kStepCh];
+    T B[kStepRows][kDState];
+    T C[kStepRows][kDState];
+};
+
+template <typename T>
+struct StepSmem {
+    StepStage<T> st[kStepStages];
+    uint64_t full[kStepStages];
+    uint64_t empty[kStepStages];
+};
+
+struct StepArgs {
+    CUtensorMap tm_state, tm_x, tm_dt, tm_z, tm_B, tm_C;
+    ScanParams p;
+    int ntiles, ntiles_d, has_gate;
+};
+
+// Lane q of a 4-lane group holds the group's shares part[0..3] (one per row of
+// the tile); return the full 4-lane sum of row q (two shuffle rounds, the
+// lanes of a group are adjacent).
+__device__ __forceinline__ float reduce_rows(const float (&part)[kStepRows], int q) {
     const bool hi = (q & 2) != 0;
     float k0 = hi ? part[2] : part[0], k1 = hi ? part[3] : part[1];
     const float s0 = hi ? part[0] : part[2], s1 = hi ? part[1] : part[3];
@@ -32,75 +60,141 @@ __device__ __forceinline__ float reduce_slots(const float (&part)[4], int q) {
     return keep + __shfl_xor_sync(kFull, send, 1);
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// Four consecutive shared-memory elements of the input dtype, widened.
+__device__ __forceinline__ float4 lds4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
+__device__ __forceinline__ float4 lds4(const __nv_bfloat16 *p) {
+    const uint2 u = *reinterpret_cast<const uint2 *>(p);
+    return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                       __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+}
+
 // ---------------------------------------------------------------------------
 // mb_step: state[b, d, :] <- one recurrence step (Eq. 2 with L = 1), y[b, 0, d].
-// Lane (g, q) of a warp: slot j covers channel wbase + 8 j + g, states 4q..4q+3.
-// The lane computes the channel scalars (Delta, Delta*x, D*x, silu z) only for
-// slot q and hands Delta, Delta*x to its group by shuffle; after the 4-lane
-// reduction it also owns slot q's output.
+// Persistent, warp-specialised streaming kernel. The work is cut into tiles
+// of 64 channels x 4 batch rows (16 KB of state); CTA i takes tiles i, i + grid,
+// ... A producer warp streams each tile's state, x, dt, z, B and C into a
+// kStepStages-deep shared-memory ring with TMA; 8 consumer warps compute it.
+// Consumer lane (g, q) of warp w serves channel d0 + 8 w + g, states 4q..4q+3,
+// for the tile's 4 rows; lane q evaluates the channel scalars (Delta, Delta*x,
+// D*x, silu z) of row q only and shares Delta, Delta*x by shuffle, and after
+// the 4-lane reduction owns row q's output. New states go straight from
+// registers to global memory (512 contiguous bytes per warp and row).
 template <typename T>
-__global__ void __launch_bounds__(kStepThreads, 4) step_kernel(ScanParams p) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int g = lane >> 2, q = lane & 3;
+__global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constant__ StepArgs a) {
+    extern __shared__ unsigned char smem_dyn[];
+    StepSmem<T> &s = *reinterpret_cast<StepSmem<T> *>(
+        (reinterpret_cast<uintptr_t>(smem_dyn) + 127) & ~static_cast<uintptr_t>(127));
+    const ScanParams &p = a.p;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t D = p.d_inner;
-    const int64_t nchan = p.batch * D;
-    const int64_t wbase = (int64_t)blockIdx.x * kStepChPerCta + warp * kStepChPerWarp;
-    const T *x = static_cast<const T *>(p.x);
-    const T *z = static_cast<const T *>(p.z);
-    const T *dt = static_cast<const T *>(p.dt);
-    const T *Bm = static_cast<const T *>(p.B);
-    const T *Cm = static_cast<const T *>(p.C);
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kStepStages; ++i) {
+            mbar_init(&s.full[i], 1);
+            mbar_init(&s.empty[i], kStepConsumers);
+        }
+        fence_mbar_init();
+    }
+    __syncthreads();
+
+    if (warp == kStepConsumers) {
+        // ---- producer
+        if (lane == 0) {
+            constexpr uint32_t st_bytes = kStepRows * kStepCh * kDState * 4;
+            constexpr uint32_t tok = kStepRows * kStepCh * sizeof(T), bc = kStepRows * kDState * sizeof(T);
+            const uint32_t bytes = st_bytes + (a.has_gate ? 3 : 2) * tok + 2 * bc;
+            for (int j = 0;; ++j) {
+                const int k = blockIdx.x + j * gridDim.x;
+                if (k >= a.ntiles) break;
+                const int si = j % kStepStages;
+                if (j >= kStepStages &&
+                    !mbar_wait(&s.empty[si], (uint32_t)((j / kStepStages - 1) & 1))) {
+                    report(p.status, 4 /* MB_ERR_TIMEOUT */, k);
+                    break;
+                }
+                const int d0 = (k % a.ntiles_d) * kStepCh, b0 = (k / a.ntiles_d) * kStepRows;
+                StepStage<T> &t = s.st[si];
+                mbar_arrive_expect_tx(&s.full[si], bytes);
+                tma_load_3d(&t.state[0][0][0], &a.tm_state, &s.full[si], 0, d0, b0);
+                tma_load_2d(&t.x[0][0], &a.tm_x, &s.full[si], d0, b0);
+                tma_load_2d(&t.dt[0][0], &a.tm_dt, &s.full[si], d0, b0);
+                if (a.has_gate) tma_load_2d(&t.z[0][0], &a.tm_z, &s.full[si], d0, b0);
+                tma_load_2d(&t.B[0][0], &a.tm_B, &s.full[si], 0, b0);
+                tma_load_2d(&t.C[0][0], &a.tm_C, &s.full[si], 0, b0);
+            }
+        }
+        return;
+    }
+
+    // ---- consumers
+    const int g = lane >> 2, q = lane & 3;
+    const int c = warp * 8 + g;
     float4 *state = reinterpret_cast<float4 *>(p.h_out);
-
-    float4 h[kSlots];
+    T *y = static_cast<T *>(p.y);
+    int64_t cur_d0 = -1;
+    float2 a01 = make_float2(0.f, 0.f), a23 = a01;
+    float bias = 0.f, dsk = 0.f;
+    for (int j = 0;; ++j) {
+        const int k = blockIdx.x + j * gridDim.x;
+        if (k >= a.ntiles) break;
+        const int si = j % kStepStages;
+        if (!mbar_wait(&s.full[si], (uint32_t)((j / kStepStages) & 1))) {
+            if (lane == 0) report(p.status, 4 /* MB_ERR_TIMEOUT */, k);
+            break;
+        }
+        const int64_t d0 = (int64_t)(k % a.ntiles_d) * kStepCh, b0 = (int64_t)(k / a.ntiles_d) * kStepRows;
+        const int64_t d = d0 + c;
+        const bool dok = d < D;
+        if (d0 != cur_d0) {
+            cur_d0 = d0;
+            const int64_t dd = dok ? d : 0;
+            const float4 av = ldg4(p.A + dd * kDState + 4 * q);
+            a01 = make_float2(av.x * kLog2e, av.y * kLog2e);
+            a23 = make_float2(av.z * kLog2e, av.w * kLog2e);
+            bias = (dok && p.dt_bias) ? __ldg(p.dt_bias + dd) : 0.f;
+            dsk = (dok && p.D) ? __ldg(p.D + dd) : 0.f;
+        }
+        const StepStage<T> &t = s.st[si];
+        float4 h[kStepRows];
 #pragma unroll
-    for (int j = 0; j < kSlots; ++j) {
-        const int64_t ch = wbase + 8 * j + g;
-        h[j] = ch < nchan ? __ldcs(state + ch * (kDState / 4) + q) : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-
-    // channel scalars of slot q
-    const int64_t mc = wbase + 8 * q + g;
-    const bool mok = mc < nchan;
-    const int64_t md = mok ? mc % D : 0;
-    float delta = 0.f, gx = 0.f, xd = 0.f, sz = 1.f;
-    if (mok) {
-        const float xv = ldg1(x + mc);
-        delta = softplus(ldg1(dt + mc) + (p.dt_bias ? __ldg(p.dt_bias + md) : 0.f));
-        gx = delta * xv;
-        xd = (p.D ? __ldg(p.D + md) : 0.f) * xv;
-        if (z) sz = silu(ldg1(z + mc));
-    }
-
-    float part[kSlots];
+        for (int u = 0; u < kStepRows; ++u) h[u] = lds4(&t.state[u][c][4 * q]);
+        // channel scalars of row q
+        const float xv = to_f32(t.x[q][c]);
+        const float delta = softplus(to_f32(t.dt[q][c]) + bias);
+        const float gx = delta * xv, xd = dsk * xv;
+        const float sz = a.has_gate ? silu(to_f32(t.z[q][c])) : 1.f;
+        float part[kStepRows];
 #pragma unroll
-    for (int j = 0; j < kSlots; ++j) {
-        const int64_t ch = wbase + 8 * j + g;
-        const int64_t cch = ch < nchan ? ch : 0;
-        const int64_t b = cch / D, d = cch - b * D;
-        const float dj = __shfl_sync(kFull, delta, 4 * g + j);
-        const float gj = __shfl_sync(kFull, gx, 4 * g + j);
-        const float4 av = ldg4(p.A + d * kDState + 4 * q);
-        const float4 bv = ldg4(Bm + b * kDState + 4 * q);
-        const float4 cv = ldg4(Cm + b * kDState + 4 * q);
-        float2 h01 = make_float2(h[j].x, h[j].y), h23 = make_float2(h[j].z, h[j].w);
-        const float2 dd = make_float2(dj, dj), gg = make_float2(gj, gj);
-        const float2 e01 = mul2(dd, make_float2(av.x * kLog2e, av.y * kLog2e));
-        const float2 e23 = mul2(dd, make_float2(av.z * kLog2e, av.w * kLog2e));
-        h01 = fma2(make_float2(ex2(e01.x), ex2(e01.y)), h01, mul2(make_float2(bv.x, bv.y), gg));
-        h23 = fma2(make_float2(ex2(e23.x), ex2(e23.y)), h23, mul2(make_float2(bv.z, bv.w), gg));
-        h[j] = make_float4(h01.x, h01.y, h23.x, h23.y);
-        const float2 acc = fma2(make_float2(cv.z, cv.w), h23, mul2(make_float2(cv.x, cv.y), h01));
-        part[j] = acc.x + acc.y;
-    }
-    const float ysum = reduce_slots(part, q);
-
+        for (int u = 0; u < kStepRows; ++u) {
+            const int src = (lane & ~3) | u;
+            const float du = __shfl_sync(kFull, delta, src);
+            const float gu = __shfl_sync(kFull, gx, src);
+            const float4 bv = lds4(&t.B[u][4 * q]);
+            const float4 cv = lds4(&t.C[u][4 * q]);
+            const float2 dd2 = make_float2(du, du), gg = make_float2(gu, gu);
+            const float2 e01 = mul2(dd2, a01), e23 = mul2(dd2, a23);
+            float2 h01 = make_float2(h[u].x, h[u].y), h23 = make_float2(h[u].z, h[u].w);
+            h01 = fma2(make_float2(ex2(e01.x), ex2(e01.y)), h01, mul2(make_float2(bv.x, bv.y), gg));
+            h23 = fma2(make_float2(ex2(e23.x), ex2(e23.y)), h23, mul2(make_float2(bv.z, bv.w), gg));
+            h[u] = make_float4(h01.x, h01.y, h23.x, h23.y);
+            const float2 acc = fma2(make_float2(cv.z, cv.w), h23, mul2(make_float2(cv.x, cv.y), h01));
+            part[u] = acc.x + acc.y;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s.empty[si]);   // this warp is done with the stage
 #pragma unroll
-    for (int j = 0; j < kSlots; ++j) {
-        const int64_t ch = wbase + 8 * j + g;
-        if (ch < nchan) __stcs(state + ch * (kDState / 4) + q, h[j]);
+        for (int u = 0; u < kStepRows; ++u) {
+            const int64_t b = b0 + u;
+            if (dok && b < p.batch) __stcs(state + (b * D + d) * (kDState / 4) + q, h[u]);
+        }
+        const float ysum = reduce_rows(part, q);
+        const int64_t b = b0 + q;
+        if (dok && b < p.batch) y[b * D + d] = from_f32<T>((ysum + xd) * sz);
     }
-    if (mok) static_cast<T *>(p.y)[mc] = from_f32<T>((ysum + xd) * sz);
 }
 
 // ---------------------------------------------------------------------------
@@ -131,17 +225,54 @@ rollback_kernel(const float4 *h0 /* may alias h_out */, const float4 *__restrict
     for (int u = 0; u < kRbVec; ++u) h_out[i0 + u] = v[u];
 }
 
+template <typename T>
+cudaError_t launch_step_typed(const ScanParams &p, cudaStream_t s) {
+    const int es = sizeof(T);
+    StepArgs a;
+    memset(&a, 0, sizeof(a));
+    a.p = p;
+    a.has_gate = p.z != nullptr;
+    a.ntiles_d = (int)((p.d_inner + kStepCh - 1) / kStepCh);
+    a.ntiles = a.ntiles_d * (int)((p.batch + kStepRows - 1) / kStepRows);
+    const uint64_t sdims[3] = {kDState, (uint64_t)p.d_inner, (uint64_t)p.batch};
+    const uint64_t sstr[2] = {kDState * 4, (uint64_t)p.d_inner * kDState * 4};
+    const uint32_t sbox[3] = {kDState, kStepCh, kStepRows};
+    const uint64_t tdims[2] = {(uint64_t)p.d_inner, (uint64_t)p.batch};
+    const uint64_t tstr[1] = {(uint64_t)p.d_inner * es};
+    const uint32_t tbox[2] = {kStepCh, kStepRows};
+    const uint64_t bdims[2] = {kDState, (uint64_t)p.batch};
+    const uint64_t bstr[1] = {(uint64_t)kDState * es};
+    const uint32_t bbox[2] = {kDState, kStepRows};
+    if (!encode_tmap(&a.tm_state, p.h_out, 4, 3, sdims, sstr, sbox) ||
+        !encode_tmap(&a.tm_x, p.x, es, 2, tdims, tstr, tbox) ||
+        !encode_tmap(&a.tm_dt, p.dt, es, 2, tdims, tstr, tbox) ||
+        (p.z && !encode_tmap(&a.tm_z, p.z, es, 2, tdims, tstr, tbox)) ||
+        !encode_tmap(&a.tm_B, p.B, es, 2, bdims, bstr, bbox) ||
+        !encode_tmap(&a.tm_C, p.C, es, 2, bdims, bstr, bbox))
+        return cudaErrorInvalidValue;
+    const size_t smem = sizeof(StepSmem<T>) + 128;
+    auto k = step_kernel<T>;
+    static int ctas = 0;   // resident CTAs per SM x SMs, computed once per process
+    if (ctas == 0) {
+        cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        int dev = 0, sms = 0, per = 0;
+        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k, kStepThreads, smem)) != cudaSuccess)
+            return e;
+        ctas = sms * (per > 0 ? per : 1);
+    }
+    const int grid = a.ntiles < ctas ? a.ntiles : ctas;
+    k<<<grid, kStepThreads, smem, s>>>(a);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_step(const ScanParams &p, bool bf16, cudaStream_t s) {
-    const int64_t nchan = p.batch * p.d_inner;
-    const int64_t grid = (nchan + kStepChPerCta - 1) / kStepChPerCta;
-    if (grid == 0) return cudaSuccess;
-    if (bf16)
-        step_kernel<__nv_bfloat16><<<(unsigned)grid, kStepThreads, 0, s>>>(p);
-    else
-        step_kernel<float><<<(unsigned)grid, kStepThreads, 0, s>>>(p);
-    return cudaGetLastError();
+    if (p.batch == 0 || p.d_inner == 0) return cudaSuccess;
+    return bf16 ? launch_step_typed<__nv_bfloat16>(p, s) : launch_step_typed<float>(p, s);
 }
 
 cudaError_t launch_rollback(const float *h0, const float *h_all, const int32_t *accept,

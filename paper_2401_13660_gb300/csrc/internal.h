@@ -2,6 +2,7 @@
 // kernels. Plain C++ structs of device pointers and sizes; no torch types.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -26,6 +27,12 @@ struct ScanParams {
 };
 
 constexpr int kDState = 16;
+
+// Encode a tiled TMA tensor map over `base` (bf16 when elem_bytes == 2, else
+// fp32): dims innermost first, strides[i] = byte stride of dimension i + 1,
+// box = tile extent per dimension. Out-of-range elements load as zeros.
+bool encode_tmap(CUtensorMap *m, const void *base, int elem_bytes, int rank, const uint64_t *dims,
+                 const uint64_t *strides, const uint32_t *box);
 
 // Launchers: return the cudaError_t of the launch.
 cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s);

@@ -348,41 +348,16 @@ __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant
 }
 
 // ---------------------------------------------------------------------------
-// Host side: tensor maps (encoded per call through the driver entry point, so
-// the library does not link libcuda) and the launch.
-using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
-                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
-                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-    static EncodeTiledFn fn = [] {
-        void *f = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
-                                             &q) != cudaSuccess ||
-            q != cudaDriverEntryPointSuccess)
-            f = nullptr;
-        return reinterpret_cast<EncodeTiledFn>(f);
-    }();
-    return fn;
-}
+// Host side: tensor maps and the launch.
 
 // [batch, L, inner] tensor with a (box_inner x kT x 1) box.
 bool make_map(CUtensorMap *m, const void *base, bool bf16, int64_t batch, int64_t L, int64_t inner,
               int box_inner) {
-    EncodeTiledFn enc = encode_fn();
-    if (!enc) return false;
     const int64_t es = bf16 ? 2 : 4;
-    cuuint64_t dims[3] = {(cuuint64_t)inner, (cuuint64_t)L, (cuuint64_t)batch};
-    cuuint64_t strides[2] = {(cuuint64_t)(inner * es), (cuuint64_t)(L * inner * es)};
-    cuuint32_t box[3] = {(cuuint32_t)box_inner, (cuuint32_t)kT, 1};
-    cuuint32_t estr[3] = {1, 1, 1};
-    CUresult r = enc(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3,
-                     const_cast<void *>(base), dims, strides, box, estr,
-                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
+    const uint64_t dims[3] = {(uint64_t)inner, (uint64_t)L, (uint64_t)batch};
+    const uint64_t strides[2] = {(uint64_t)(inner * es), (uint64_t)(L * inner * es)};
+    const uint32_t box[3] = {(uint32_t)box_inner, (uint32_t)kT, 1};
+    return encode_tmap(m, base, (int)es, 3, dims, strides, box);
 }
 
 template <typename T, int LPC, int STAGES, bool kStoreAll>
