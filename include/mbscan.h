@@ -144,6 +144,34 @@ mb_status mb_step(const mb_scan_args *args, float *state, void *stream);
  */
 mb_status mb_check(void *ws, void *stream, int64_t *detail);
 
+/*
+ * mb_scan_prefill without a caller-provided workspace. (An addition of this
+ * library; the paper has no counterpart.)
+ *
+ * Some callers cannot allocate device memory at the point where they run the
+ * scan: code recorded into a CUDA graph or running under an allocator that
+ * owns all device memory, real-time paths that must not allocate after
+ * start-up, or plugins that are handed only input and output buffers. This
+ * entry point computes exactly what mb_scan_prefill computes, for the same
+ * arguments, but its scratch (the status block of bounded device-side
+ * waits, 256 bytes) is a fixed array inside the library, one per GPU, kept
+ * for as long as the library is loaded. It calls no allocator.
+ *
+ *  - Arguments, layouts and h_last rules are those of mb_scan_prefill.
+ *  - A problem whose workspace would exceed the fixed 256-byte array is
+ *    rejected with MB_ERR_UNSUPPORTED before anything is launched (no
+ *    supported shape needs more today).
+ *  - The first call on each GPU looks up the array's device address with that
+ *    GPU current; make that first call outside any stream capture.
+ *  - Every call clears the array on `stream` before the launch. All calls on
+ *    one GPU share the one array, so calls that may run at the same time on
+ *    the GPU (different streams without ordering) race on it; order them.
+ *  - A device-side timeout is recorded in that internal array; it cannot be
+ *    read back through mb_check (use mb_scan_prefill with a workspace when
+ *    the status matters).
+ */
+mb_status mb_scan_prefill_noalloc(const mb_scan_args *args, float *h_last, void *stream);
+
 /* Human-readable name of a status code (static string). */
 const char *mb_status_string(mb_status s);
 

@@ -5,6 +5,8 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <mutex>
+
 #include "../../include/mbscan.h"
 #include "internal.h"
 
@@ -209,3 +211,79 @@ const char *mb_status_string(mb_status s) {
 const char *mb_version(void) { return "mbscan 0.1.0 sm_103a"; }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free prefill (mb_scan_prefill_noalloc).
+//
+// The prefill kernel needs a small block of device scratch (the status block
+// that its bounded waits write). Normally the caller provides it as `ws`. For
+// callers that may not allocate device memory, this file owns one fixed
+// scratch array per device instead: a file-scope __device__ array of
+// kNoAllocScratchBytes. Host code must never hand the array's name to a
+// kernel (on the host it is only a stand-in symbol); its device address is
+// looked up once per device with cudaGetSymbolAddress while that device is
+// current, and that address is what the kernel receives. The array lives for
+// as long as the library is loaded on the device and keeps the previous
+// call's contents, so every call clears it first on its stream.
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = 256;   // the largest workspace it can stand in for
+constexpr int kNoAllocMaxDevices = 64;
+
+}  // namespace
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+namespace {
+
+std::mutex g_noalloc_mutex;
+void *g_noalloc_addr[kNoAllocMaxDevices];   // device address of the array, per device
+
+// Device address of g_noalloc_scratch on the current device, looked up on
+// the first call for that device.
+mb_status noalloc_scratch(void **out) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) return MB_ERR_CUDA;
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return MB_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (g_noalloc_addr[dev] == nullptr) {
+        void *addr = nullptr;
+        if (cudaGetSymbolAddress(&addr, g_noalloc_scratch) != cudaSuccess || addr == nullptr)
+            return MB_ERR_CUDA;
+        g_noalloc_addr[dev] = addr;
+    }
+    *out = g_noalloc_addr[dev];
+    return MB_OK;
+}
+
+// Same checks on h_last as mb_scan_prefill.
+mb_status check_h_last(const mb_scan_args *args, const float *h_last) {
+    if (!h_last) return MB_OK;
+    if (!aligned16(h_last)) return MB_ERR_INVALID_ARG;
+    const int64_t sbytes = args->batch * args->d_inner * args->d_state * 4;
+    const Range rh = range_of(h_last, sbytes);
+    if (args->h0 != h_last && overlap(rh, range_of(args->h0, sbytes))) return MB_ERR_INVALID_ARG;
+    const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
+    const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
+    if (overlap(rh, range_of(args->y, tok)) || overlap(rh, range_of(args->x, tok)) ||
+        overlap(rh, range_of(args->dt, tok)) || overlap(rh, range_of(args->z, tok)))
+        return MB_ERR_INVALID_ARG;
+    return MB_OK;
+}
+
+}  // namespace
+
+extern "C" mb_status mb_scan_prefill_noalloc(const mb_scan_args *args, float *h_last, void *stream) {
+    mb_status st = check_args(args, false);
+    if (st != MB_OK) return st;
+    if ((st = check_h_last(args, h_last)) != MB_OK) return st;
+    const size_t need = mb_workspace_size(args);
+    if (need > kNoAllocScratchBytes) return MB_ERR_UNSUPPORTED;   // larger than the fixed scratch
+    if (args->batch * args->d_inner == 0) return MB_OK;
+    void *scratch = nullptr;
+    if ((st = noalloc_scratch(&scratch)) != MB_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (need > 0 && cudaMemsetAsync(scratch, 0, need, s) != cudaSuccess) return MB_ERR_CUDA;
+    ScanParams p = to_params(args, h_last, static_cast<StatusBlock *>(scratch));
+    return from_cuda(mbscan::launch_prefill(p, args->dtype == MB_BF16, s));
+}
