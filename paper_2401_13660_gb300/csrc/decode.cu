@@ -19,7 +19,10 @@ constexpr int kStepConsumers = 8;                          // consumer warps
 constexpr int kStepThreads = 32 * (kStepConsumers + 1);    // + one producer warp
 constexpr int kStepCh = 8 * kStepConsumers;                // 64 channels per tile
 constexpr int kStepRows = 4;                               // batch rows per tile
-constexpr int kStepStages = 4;
+#ifndef MB_STEP_STAGES
+#define MB_STEP_STAGES 4
+#endif
+constexpr int kStepStages = MB_STEP_STAGES;
 
 // One tile of the decode step in shared memory (TMA destinations; every member
 // offset is a multiple of 128 bytes for both dtypes).

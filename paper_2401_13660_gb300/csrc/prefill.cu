@@ -11,8 +11,8 @@
 // and step); the associative operator of Section 2 is only needed to split a
 // span, which the h0 / h_last interface does across calls.
 //
-// A CTA (4 warps) owns CH = 128 / LPC channels of one batch row for the whole
-// span. LPC lanes share a channel, each keeping 16 / LPC of its fp32 states in
+// A CTA of kWarps warps owns CH = 32 kWarps / LPC channels of one batch row
+// for the whole span (small CTAs spread the channels evenly over the SMs). LPC lanes share a channel, each keeping 16 / LPC of its fp32 states in
 // registers. The state index varies slowest across a warp, so the 8 lanes of
 // each quarter-warp read the same B, C values (a shared-memory broadcast).
 //
@@ -21,17 +21,19 @@
 //    dt, x, z [kT x CH] and B, C [kT x 16], one mbarrier per stage (bounded
 //    waits, tma.cuh);
 //  * the CTA converts a chunk once per (t, channel) into fp32 in shared
-//    memory: (Delta, Delta*x) with Delta = softplus(dt + bias), (D*x,
-//    silu(z)), and B, C;
+//    memory: (Delta, Delta*x) with Delta = softplus(dt + bias), (D*x, silu z);
 //  * each lane scans the chunk: Abar = 2^(Delta * A*log2 e) on the SFU for all
 //    kT steps, then h = Abar*h + B*(Delta*x) and its share of C.h in packed
-//    f32x2 arithmetic; groups of LPC steps are reduced across the LPC lanes
-//    of a channel with log2(LPC) shuffle rounds, each lane finishing one
+//    f32x2 arithmetic, reading B and C straight from the TMA tile in the input
+//    dtype (for bf16 this halves the shared-memory bytes of the scan, whose
+//    bandwidth is its limit); groups of LPC steps are reduced across the LPC
+//    lanes of a channel with log2(LPC) shuffle rounds, each lane finishing one
 //    output y = (C.h + D*x) * silu(z), which goes to a shared-memory tile that
 //    one thread writes out with a TMA store.
 //  Loop iteration i converts chunk i+1 and scans chunk i in one basic block,
 //  so every warp has two independent instruction streams to interleave; one
-//  CTA barrier per chunk orders them.
+//  CTA barrier per chunk orders them, after which the stage of chunk i is
+//  refilled with chunk i + STAGES.
 // Steps at or beyond L are converted with Delta = 0, which leaves h unchanged.
 #include <string.h>
 
@@ -42,7 +44,11 @@ namespace mbscan {
 namespace {
 
 constexpr int kT = 16;            // time steps per chunk
-constexpr int kThreads = 128;     // 4 warps
+#ifndef MB_PREFILL_WARPS
+#define MB_PREFILL_WARPS 4
+#endif
+constexpr int kWarps = MB_PREFILL_WARPS;   // warps per CTA
+constexpr int kThreads = 32 * kWarps;
 #ifndef MB_PREFILL_LPC
 #define MB_PREFILL_LPC 4
 #endif
@@ -56,7 +62,7 @@ struct Geom {
     static constexpr int kSPL = kDState / LPC;     // states per lane
     static constexpr int kPairs = kSPL / 2;        // float2 state pairs per lane
     static constexpr int kChPerWarp = 32 / LPC;
-    static constexpr int kCh = 4 * kChPerWarp;     // channels per CTA
+    static constexpr int kCh = kWarps * kChPerWarp;  // channels per CTA
 };
 
 template <typename T, int CH>
@@ -72,7 +78,6 @@ template <int CH>
 struct Conv {
     float2 dg[kT][CH];          // (Delta, Delta*x)
     float2 xs[kT][CH];          // (D*x, silu(z)); silu(z) = 1 without a gate
-    float bc[kT][2 * kDState];  // B[0..15], C[0..15]
 };
 
 template <typename T, int CH, int STAGES>
@@ -112,6 +117,14 @@ __device__ __forceinline__ float2 ld_pair(const __nv_bfloat16 *p) {
     return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
 }
 
+// Four adjacent elements of the input dtype from shared memory, widened.
+__device__ __forceinline__ float4 ld_quad(const float *p) { return *reinterpret_cast<const float4 *>(p); }
+__device__ __forceinline__ float4 ld_quad(const __nv_bfloat16 *p) {
+    const uint2 u = *reinterpret_cast<const uint2 *>(p);
+    return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                       __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+}
+
 // Per-thread constants of the conversion role: thread converts the adjacent
 // channel pair (2 cp, 2 cp + 1) at steps th, th + kRows, ...
 template <int CH>
@@ -124,7 +137,7 @@ struct ConvRole {
     bool ok;
 };
 
-// Convert one chunk: raw TMA tiles -> fp32 (Delta, Delta*x), (D*x, silu z), B, C.
+// Convert one chunk: raw TMA tiles -> fp32 (Delta, Delta*x), (D*x, silu z).
 template <typename T, int CH>
 __device__ __forceinline__ void convert(Conv<CH> &cv, const Raw<T, CH> &r, const ConvRole<CH> &cr,
                                         int64_t t0, int64_t L, bool gate) {
@@ -148,12 +161,6 @@ __device__ __forceinline__ void convert(Conv<CH> &cv, const Raw<T, CH> &r, const
         }
         *reinterpret_cast<float4 *>(&cv.dg[t][c]) = dg;
         *reinterpret_cast<float4 *>(&cv.xs[t][c]) = xs;
-    }
-    {   // B, C: kT steps x 32 values, 4 per thread
-        const int t = threadIdx.x >> 3, k4 = (threadIdx.x & 7) * 4;
-        const T *src = k4 < kDState ? &r.B[t][k4] : &r.C[t][k4 - kDState];
-        const float2 lo = ld_pair(src), hi = ld_pair(src + 2);
-        *reinterpret_cast<float4 *>(&cv.bc[t][k4]) = make_float4(lo.x, lo.y, hi.x, hi.y);
     }
 }
 
@@ -247,10 +254,6 @@ __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant
         }
         return;
     }
-    if (tid == 0 && STAGES < nchunks) {
-        fence_proxy_async_smem();
-        issue_chunk(s, a, 0, STAGES, d0, b);
-    }
 
     for (int64_t i = 0; i < nchunks; ++i) {
         const int64_t t0 = i * kT;
@@ -262,6 +265,7 @@ __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant
 
         // (2) chunk i: decays of all kT steps, recurrence, shares of C.h
         const Conv<CH> &cv = s.cv[i & 1];
+        const Raw<T, CH> &rs = s.raw[i % STAGES];   // B, C straight from the TMA tile
         float2 ab[kT][G::kPairs];
         float gx[kT];
 #pragma unroll
@@ -282,8 +286,8 @@ __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant
             float2 bp[G::kPairs], cp[G::kPairs];
 #pragma unroll
             for (int k = 0; k < G::kPairs; k += 2) {
-                const float4 b4 = *reinterpret_cast<const float4 *>(&cv.bc[t][G::kSPL * q + 2 * k]);
-                const float4 c4 = *reinterpret_cast<const float4 *>(&cv.bc[t][kDState + G::kSPL * q + 2 * k]);
+                const float4 b4 = ld_quad(&rs.B[t][G::kSPL * q + 2 * k]);
+                const float4 c4 = ld_quad(&rs.C[t][G::kSPL * q + 2 * k]);
                 bp[k] = make_float2(b4.x, b4.y); bp[k + 1] = make_float2(b4.z, b4.w);
                 cp[k] = make_float2(c4.x, c4.y); cp[k + 1] = make_float2(c4.z, c4.w);
             }
@@ -323,7 +327,7 @@ __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant
         if (__syncthreads_or(ok ? 0 : 1)) {
             if (tid == 0) {
                 report(p.status, 4 /* MB_ERR_TIMEOUT */, i + 1);
-                for (int64_t j = i + 1; j < i + 1 + STAGES && j < nchunks; ++j)
+                for (int64_t j = i + 1; j < i + STAGES && j < nchunks; ++j)
                     mbar_wait(&s.full[j % STAGES], (uint32_t)((j / STAGES) & 1));
                 bulk_wait_all();
             }
@@ -332,9 +336,11 @@ __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant
         if (tid == 0) {
             tma_store_3d(&a.tm_y, &ys[0][0], d0, (int)t0, b);
             bulk_commit();
-            if (has_next && i + 1 + STAGES < nchunks) {
+            // stage i % STAGES (chunk i: converted last iteration, scanned
+            // now) is free: refill it with chunk i + STAGES
+            if (i + STAGES < nchunks) {
                 fence_proxy_async_smem();
-                issue_chunk(s, a, nst, i + 1 + STAGES, d0, b);
+                issue_chunk(s, a, (int)(i % STAGES), i + STAGES, d0, b);
             }
         }
     }

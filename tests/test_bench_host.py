@@ -1,0 +1,72 @@
+"""CPU checks of bench.py's host logic: algorithmic byte counts and the
+multi-rank timing reduction (two gloo ranks on 127.0.0.1)."""
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+import bench
+
+
+def test_algorithmic_bytes_of_the_workloads():
+    # Read + write bytes, each tensor once (prefill 353M-shaped, verify, rollback,
+    # decode step per layer).
+    assert sum(bench.bytes_prefill(8, 8192, 2048)) == 1_079_132_160
+    assert sum(bench.bytes_prefill(4, 8192, 3584, h0=True)) == 943_714_304
+    assert sum(bench.bytes_verify(32, 16, 2048)) == 79_872_000
+    assert sum(bench.bytes_rollback(32, 2048)) == 8_388_736
+    assert sum(bench.bytes_step(256, 4608)) == 160_780_288
+    parts = bench.step_bytes()
+    assert parts["step"] == 48 * 160_780_288
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        out[rank] = bench.reduce_max(10.0 + rank, dist)
+    finally:
+        dist.destroy_process_group()
+
+
+def test_reduce_max_over_two_gloo_ranks():
+    ctx = mp.get_context("spawn")
+    with ctx.Manager() as m:
+        out = m.dict()
+        port = _free_port()
+        procs = [ctx.Process(target=_worker, args=(r, 2, port, out)) for r in range(2)]
+        for p in procs:
+            p.start()
+        for p in procs:
+            p.join(120)
+            assert p.exitcode == 0
+        assert dict(out) == {0: 11.0, 1: 11.0}
+
+
+def test_reduce_max_single_process_is_identity():
+    assert bench.reduce_max(3.5, None) == 3.5
+
+
+def test_traffic_record_needs_matching_source(tmp_path, monkeypatch):
+    (tmp_path / "profiles").mkdir()
+    src = tmp_path / "paper_2401_13660_gb300" / "csrc"
+    src.mkdir(parents=True)
+    (src / "k.cu").write_text("kernel source v1\n")
+    import hashlib
+    sha = hashlib.sha256(b"kernel source v1\n").hexdigest()[:16]
+    (tmp_path / "profiles" / "ncu_traffic.txt").write_text(
+        f"kernel=my_kernel source=k.cu sha={sha} bytes_per_launch=1000\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.traffic_from_profiles("my_kernel") == 1000.0
+    (src / "k.cu").write_text("kernel source v2\n")
+    assert bench.traffic_from_profiles("my_kernel") is None
+    assert bench.traffic_from_profiles("other") is None
