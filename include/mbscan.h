@@ -127,6 +127,24 @@ mb_status mb_rollback(const float *h0, const float *h_all, const int32_t *accept
                       void *stream);
 
 /*
+ * Bifurcation test of speculative decoding (Algorithm 1): how many leading
+ * drafted bytes of each stream are among the verifier's top-beta candidates.
+ *   logits  : [streams, k, 256], dtype (MB_F32 or MB_BF16); row (s, i) is the
+ *             verifier's next-byte score for drafted position i of stream s
+ *             (the p_i of Algorithm 1, up to a monotone map)
+ *   drafted : [streams, k] uint8, the drafted bytes
+ *   beta    : >= 1; rank(b) = 1 + #{v : logit[v] > logit[b]} (ties share the
+ *             better rank, a NaN score is never larger); byte i is accepted
+ *             when rank <= beta
+ *   accept  : [streams] int32 output, the index of the first drafted byte that
+ *             is not accepted, or k when all are; this is the accept count
+ *             that mb_rollback takes.
+ * Device pointers; logits 16-byte aligned.
+ */
+mb_status mb_accept_topk(const void *logits, int32_t dtype, const uint8_t *drafted, int64_t streams,
+                         int64_t k, int32_t beta, int32_t *accept, void *stream);
+
+/*
  * One recurrent decode step (Section 6.3: generation runs the recurrence
  * directly, one byte per call). args->seqlen must be 1; args->h0 is ignored.
  * `state` [batch, d_inner, d_state] fp32 is read and updated in place; y is

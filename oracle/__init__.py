@@ -12,6 +12,8 @@ Functions (MambaByte, Eq. 2-3, discretisation appendix, Table 6, Algorithm 1):
                  optionally every per-position state (verify).
 * ``step``     - one recurrent decode step (a scan of length 1).
 * ``rollback`` - keep the state after ``accept`` drafted bytes.
+* ``accept_topk`` - Algorithm 1's bifurcation: leading drafted bytes whose
+                 rank in the verifier's distribution is within top-beta.
 
 Inputs are widened exactly to float64 before the call (bf16 and fp32 values
 are exactly representable in fp64).
@@ -130,4 +132,29 @@ def rollback(h0, h_all, accept):
                                  acc.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), _ptr(out))
     if rc != 0:
         raise RuntimeError("oracle_rollback: accept count out of [0, k]")
+    return out
+
+
+def accept_topk(logits, drafted, beta):
+    """Accept count per stream (Algorithm 1, bifurcation position): the number
+    of leading drafted bytes b_i with rank_{p_i}(b_i) <= beta, where
+    rank(b) = 1 + #{v : score[v] > score[b]}. logits [streams, k, 256],
+    drafted [streams, k]. Plain loops over streams and positions."""
+    if hasattr(logits, "detach"):
+        logits = logits.detach().to("cpu").double().numpy()
+    if hasattr(drafted, "detach"):
+        drafted = drafted.detach().to("cpu").numpy()
+    logits = np.asarray(logits, dtype=np.float64)
+    drafted = np.asarray(drafted)
+    streams, k, _ = logits.shape
+    out = np.empty(streams, dtype=np.int32)
+    for s in range(streams):
+        a = k
+        for i in range(k):
+            row = logits[s, i]
+            rank = 1 + int(np.sum(row > row[int(drafted[s, i])]))
+            if rank > beta:
+                a = i
+                break
+        out[s] = a
     return out

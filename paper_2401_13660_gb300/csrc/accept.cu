@@ -1,0 +1,74 @@
+// Bifurcation of speculative decoding (MambaByte Algorithm 1): for every
+// stream, count how many leading drafted bytes fall in the verifier's top-beta
+// candidates. The count a[s] is what the rollback (and the corrector loop)
+// resumes from: the state after a[s] accepted bytes.
+//
+// rank_p(b) = 1 + #{v in 0..255 : logit[v] > logit[b]} (ties share the better
+// rank; a NaN logit is never larger). Drafted byte i is accepted when
+// rank <= beta; a[s] = the first i (0-based) that is not accepted, else k.
+//
+// One warp per stream; lane l compares the 8 logits 8l .. 8l+7 of a position
+// with the drafted byte's logit and the warp sums the counts.
+#include "common.cuh"
+
+namespace mbscan {
+namespace {
+
+__device__ __forceinline__ void load8(const float *p, float (&v)[8]) {
+    const float4 a = __ldg(reinterpret_cast<const float4 *>(p));
+    const float4 b = __ldg(reinterpret_cast<const float4 *>(p) + 1);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void load8(const __nv_bfloat16 *p, float (&v)[8]) {
+    const uint4 u = __ldg(reinterpret_cast<const uint4 *>(p));
+    const unsigned w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        v[2 * j] = __uint_as_float(w[j] << 16);
+        v[2 * j + 1] = __uint_as_float(w[j] & 0xffff0000u);
+    }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(128) accept_kernel(const T *__restrict__ logits,
+                                                     const uint8_t *__restrict__ drafted,
+                                                     int64_t streams, int64_t k, int beta,
+                                                     int32_t *__restrict__ accept) {
+    const int lane = threadIdx.x & 31;
+    const int64_t s = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+    if (s >= streams) return;   // whole warp leaves together
+    int a = (int)k;
+    for (int64_t i = 0; i < k; ++i) {
+        const T *row = logits + (s * k + i) * 256;
+        const int byte = __ldg(drafted + s * k + i);
+        const float target = to_f32(row[byte]);
+        float v[8];
+        load8(row + 8 * lane, v);
+        int greater = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) greater += v[j] > target ? 1 : 0;
+        const int rank = 1 + __reduce_add_sync(kFull, greater);
+        if (rank > beta) {   // warp-uniform
+            a = (int)i;
+            break;
+        }
+    }
+    if (lane == 0) accept[s] = a;
+}
+
+}  // namespace
+
+cudaError_t launch_accept(const void *logits, bool bf16, const uint8_t *drafted, int64_t streams,
+                          int64_t k, int beta, int32_t *accept, cudaStream_t s) {
+    if (streams == 0) return cudaSuccess;
+    const unsigned grid = (unsigned)((streams + 3) / 4);
+    if (bf16)
+        accept_kernel<__nv_bfloat16><<<grid, 128, 0, s>>>(
+            static_cast<const __nv_bfloat16 *>(logits), drafted, streams, k, beta, accept);
+    else
+        accept_kernel<float><<<grid, 128, 0, s>>>(static_cast<const float *>(logits), drafted,
+                                                  streams, k, beta, accept);
+    return cudaGetLastError();
+}
+
+}  // namespace mbscan

@@ -38,6 +38,8 @@ bool encode_tmap(CUtensorMap *m, const void *base, int elem_bytes, int rank, con
 cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s);
 cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s);
 cudaError_t launch_step(const ScanParams &p, bool bf16, cudaStream_t s);
+cudaError_t launch_accept(const void *logits, bool bf16, const uint8_t *drafted, int64_t streams,
+                          int64_t k, int beta, int32_t *accept, cudaStream_t s);
 cudaError_t launch_rollback(const float *h0, const float *h_all, const int32_t *accept,
                             float *h_out, int64_t batch, int64_t k, int64_t d_inner,
                             StatusBlock *status, cudaStream_t s);

@@ -162,6 +162,23 @@ mb_status mb_rollback(const float *h0, const float *h_all, const int32_t *accept
                                              static_cast<StatusBlock *>(ws), (cudaStream_t)stream));
 }
 
+mb_status mb_accept_topk(const void *logits, int32_t dtype, const uint8_t *drafted, int64_t streams,
+                         int64_t k, int32_t beta, int32_t *accept, void *stream) {
+    if (streams < 0 || k < 0 || beta < 1) return MB_ERR_INVALID_ARG;
+    if (dtype != MB_F32 && dtype != MB_BF16) return MB_ERR_INVALID_ARG;
+    if (streams > kMaxTokens || k > kMaxTokens || (k > 0 && streams > kMaxTokens / (256 * k)))
+        return MB_ERR_INVALID_ARG;
+    if (streams == 0) return MB_OK;
+    if (!accept || (reinterpret_cast<uintptr_t>(accept) & 3u)) return MB_ERR_INVALID_ARG;
+    if (k > 0 && (!logits || !drafted || !aligned16(logits))) return MB_ERR_INVALID_ARG;
+    const int64_t es = dtype == MB_BF16 ? 2 : 4;
+    const Range ra = range_of(accept, streams * 4);
+    if (overlap(ra, range_of(logits, streams * k * 256 * es)) || overlap(ra, range_of(drafted, streams * k)))
+        return MB_ERR_INVALID_ARG;
+    return from_cuda(mbscan::launch_accept(logits, dtype == MB_BF16, drafted, streams, k, beta, accept,
+                                           (cudaStream_t)stream));
+}
+
 mb_status mb_step(const mb_scan_args *args, float *state, void *stream) {
     mb_status st = check_args(args, true);
     if (st != MB_OK) return st;

@@ -198,8 +198,10 @@ __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant
     const ScanParams &p = a.p;
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
-    const int b = blockIdx.y;
-    const int d0 = blockIdx.x * CH;
+    // blockIdx.x = batch row * channel tiles + channel tile (no 65535 limit on batch)
+    const int ntd = (int)((p.d_inner + CH - 1) / CH);
+    const int b = blockIdx.x / ntd;
+    const int d0 = (blockIdx.x % ntd) * CH;
     const int64_t L = p.seqlen, D = p.d_inner;
     const int64_t nchunks = (L + kT - 1) / kT;
     const bool gate = a.has_gate != 0;
@@ -385,7 +387,7 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
     auto k = prefill_kernel<T, LPC, STAGES, kStoreAll>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    const dim3 grid((unsigned)((p.d_inner + kCh - 1) / kCh), (unsigned)p.batch);
+    const dim3 grid((unsigned)(((p.d_inner + kCh - 1) / kCh) * p.batch));
     k<<<grid, kThreads, smem, s>>>(a);
     return cudaGetLastError();
 }

@@ -65,7 +65,9 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
             lib.mb_rollback.argtypes = [vp, vp, vp, vp, i64, i64, i64, i64, vp, vp]
             lib.mb_step.argtypes = [ap, vp, vp]
             lib.mb_check.argtypes = [vp, vp, ctypes.POINTER(i64)]
-            for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_check"):
+            lib.mb_accept_topk.argtypes = [vp, ctypes.c_int32, vp, i64, i64, ctypes.c_int32, vp, vp]
+            for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_check",
+                      "mb_accept_topk"):
                 getattr(lib, f).restype = ctypes.c_int
             lib.mb_status_string.argtypes = [ctypes.c_int]
             lib.mb_status_string.restype = ctypes.c_char_p
@@ -196,6 +198,25 @@ def mb_step(x, dt, B, C, A, y, state, *, z=None, D=None, dt_bias=None, stream=No
     rc = load_library().mb_step(ctypes.byref(a), _ptr(state), _stream(stream))
     _check(rc, "mb_step")
     return y, state
+
+
+def mb_accept_topk(logits, drafted, beta, accept=None, stream=None):
+    """Accept counts of speculative decoding: logits [streams, k, 256] (fp32 or
+    bf16), drafted [streams, k] uint8 -> accept [streams] int32."""
+    if logits.dtype not in _DTYPES:
+        raise TypeError(f"unsupported logits dtype {logits.dtype}")
+    streams, k, v = logits.shape
+    if v != 256:
+        raise ValueError("logits must have 256 entries per position")
+    _need(logits, "logits", logits.dtype)
+    _need(drafted, "drafted", torch.uint8, (streams, k), logits.device)
+    if accept is None:
+        accept = torch.empty(streams, dtype=torch.int32, device=logits.device)
+    _need(accept, "accept", torch.int32, (streams,), logits.device)
+    rc = load_library().mb_accept_topk(_ptr(logits), _DTYPES[logits.dtype], _ptr(drafted), streams, k,
+                                       int(beta), _ptr(accept), _stream(stream))
+    _check(rc, "mb_accept_topk")
+    return accept
 
 
 def mb_check(ws, stream=None):
