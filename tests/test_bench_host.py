@@ -23,6 +23,16 @@ def test_algorithmic_bytes_of_the_workloads():
     assert parts["step"] == 48 * 160_780_288
 
 
+def test_sfu_roofline_of_the_scan():
+    # Per element: one ex2 (1/32 clk/SM); per (b, t, d): softplus (ex2 + lg2)
+    # and silu (ex2 + rcp) shared by 16 states -> (2/32 + 2/16) / 16.
+    assert bench.sfu_clocks_per_element() == pytest.approx(1 / 32 + (2 / 32 + 2 / 16) / 16)
+    r = bench.sfu_roofline(elements=2**31, seconds=1e-3, sms=152, sm_mhz=2000.0)
+    assert r["peak"] == pytest.approx(152 * 2e9 / bench.sfu_clocks_per_element())
+    assert r["achieved"] == pytest.approx(2**31 / 1e-3)
+    assert r["frac"] == pytest.approx(r["achieved"] / r["peak"], rel=1e-3)
+
+
 def _free_port():
     with socket.socket() as s:
         s.bind(("127.0.0.1", 0))
