@@ -154,6 +154,28 @@ mb_status mb_accept_topk(const void *logits, int32_t dtype, const uint8_t *draft
 mb_status mb_step(const mb_scan_args *args, float *state, void *stream);
 
 /*
+ * Resume after the bifurcation (Algorithm 1): one recurrent decode step for
+ * every stream s, starting from the state kept after accept[s] drafted bytes
+ * (args->h0[s] when accept[s] == 0, h_all[s, accept[s]-1] when
+ * 1 <= accept[s] <= k), writing the new state to state[s]. The result is that
+ * of mb_rollback(args->h0, h_all, accept, state, ...) followed by
+ * mb_step(args, state), without the rollback's own pass over the state.
+ *   args    : as for mb_step (seqlen 1); args->h0 = the cached states
+ *             [batch, d_inner, d_state] fp32, NULL = zeros
+ *   h_all   : [batch, k, d_inner, d_state] fp32, the per-position states of
+ *             the last mb_scan_verify (k >= 1)
+ *   accept  : [batch] int32 device array, values in [0, k] (mb_accept_topk)
+ *   state   : [batch, d_inner, d_state] fp32 output; may alias args->h0, not
+ *             h_all
+ *   ws      : workspace (mb_workspace_size(args) bytes, 256-byte aligned) or
+ *             NULL; an accept count outside [0, k] is a caller error: that
+ *             stream's state and y are left untouched and the first such
+ *             stream index is recorded in ws's status block (mb_check).
+ */
+mb_status mb_step_resume(const mb_scan_args *args, const float *h_all, const int32_t *accept,
+                         int64_t k, float *state, void *ws, size_t ws_bytes, void *stream);
+
+/*
  * Read and clear the status block of a workspace (blocking: waits for
  * `stream`). Returns MB_OK, or the first device-side error recorded by
  * calls on that workspace since the last mb_check. If detail != NULL it

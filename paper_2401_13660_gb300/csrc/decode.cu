@@ -45,9 +45,21 @@ struct StepSmem {
 
 struct StepArgs {
     CUtensorMap tm_state, tm_x, tm_dt, tm_z, tm_B, tm_C;
+    // resume: initial state of row s from h0 (tm_state over p.h0, box of one
+    // row) or from h_all[s, accept[s]-1] (tm_hall)
+    CUtensorMap tm_hall;
+    const int32_t *accept;
+    int64_t k;
     ScanParams p;
-    int ntiles, ntiles_d, has_gate;
+    int ntiles, ntiles_d, has_gate, has_h0;
 };
+
+// Resume: the drafted-byte index whose state row s starts from (0 .. k-1),
+// -1 for the cached state h0, or -2 when accept[s] is outside [0, k].
+__device__ __forceinline__ int resume_index(const StepArgs &a, int64_t s) {
+    const int acc = __ldg(a.accept + s);
+    return (acc < 0 || acc > a.k) ? -2 : acc - 1;
+}
 
 // Lane q of a 4-lane group holds the group's shares part[0..3] (one per row of
 // the tile); return the full 4-lane sum of row q (two shuffle rounds, the
@@ -86,7 +98,11 @@ __device__ __forceinline__ float4 lds4(const __nv_bfloat16 *p) {
 // D*x, silu z) of row q only and shares Delta, Delta*x by shuffle, and after
 // the 4-lane reduction owns row q's output. New states go straight from
 // registers to global memory (512 contiguous bytes per warp and row).
-template <typename T>
+// kResume (speculative decoding, after the bifurcation of Algorithm 1): row s
+// starts from h0[s] or h_all[s, accept[s]-1] instead of the state itself, so
+// the rollback needs no copy of its own; rows with an accept count outside
+// [0, k] are reported and left untouched.
+template <typename T, bool kResume>
 __global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constant__ StepArgs a) {
     extern __shared__ unsigned char smem_dyn[];
     StepSmem<T> &s = *reinterpret_cast<StepSmem<T> *>(
@@ -122,7 +138,20 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constan
                 const int d0 = (k % a.ntiles_d) * kStepCh, b0 = (k / a.ntiles_d) * kStepRows;
                 StepStage<T> &t = s.st[si];
                 mbar_arrive_expect_tx(&s.full[si], bytes);
-                tma_load_3d(&t.state[0][0][0], &a.tm_state, &s.full[si], 0, d0, b0);
+                if constexpr (kResume) {
+                    for (int u = 0; u < kStepRows; ++u) {
+                        const int64_t bs = b0 + u;
+                        int r = bs < p.batch ? resume_index(a, bs) : -2;
+                        if (r == -2 && bs < p.batch && d0 == 0) report(p.status, 1 /* MB_ERR_INVALID_ARG */, bs);
+                        if (r == -1 && a.has_h0)
+                            tma_load_3d(&t.state[u][0][0], &a.tm_state, &s.full[si], 0, d0, (int)bs);
+                        else   // h_all row r; r < 0 (no h0, or a row left untouched) reads zeros
+                            tma_load_4d(&t.state[u][0][0], &a.tm_hall, &s.full[si], 0, d0, r < 0 ? -1 : r,
+                                        (int)bs);
+                    }
+                } else {
+                    tma_load_3d(&t.state[0][0][0], &a.tm_state, &s.full[si], 0, d0, b0);
+                }
                 tma_load_2d(&t.x[0][0], &a.tm_x, &s.full[si], d0, b0);
                 tma_load_2d(&t.dt[0][0], &a.tm_dt, &s.full[si], d0, b0);
                 if (a.has_gate) tma_load_2d(&t.z[0][0], &a.tm_z, &s.full[si], d0, b0);
@@ -192,11 +221,15 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constan
 #pragma unroll
         for (int u = 0; u < kStepRows; ++u) {
             const int64_t b = b0 + u;
-            if (dok && b < p.batch) __stcs(state + (b * D + d) * (kDState / 4) + q, h[u]);
+            bool ok = dok && b < p.batch;
+            if constexpr (kResume) ok = ok && resume_index(a, b) != -2;
+            if (ok) __stcs(state + (b * D + d) * (kDState / 4) + q, h[u]);
         }
         const float ysum = reduce_rows(part, q);
         const int64_t b = b0 + q;
-        if (dok && b < p.batch) y[b * D + d] = from_f32<T>((ysum + xd) * sz);
+        bool yok = dok && b < p.batch;
+        if constexpr (kResume) yok = yok && resume_index(a, b) != -2;
+        if (yok) y[b * D + d] = from_f32<T>((ysum + xd) * sz);
     }
 }
 
@@ -228,12 +261,16 @@ rollback_kernel(const float4 *h0 /* may alias h_out */, const float4 *__restrict
     for (int u = 0; u < kRbVec; ++u) h_out[i0 + u] = v[u];
 }
 
-template <typename T>
-cudaError_t launch_step_typed(const ScanParams &p, cudaStream_t s) {
+template <typename T, bool kResume>
+cudaError_t launch_step_typed(const ScanParams &p, const float *h_all, const int32_t *accept, int64_t k,
+                              cudaStream_t s) {
     const int es = sizeof(T);
     StepArgs a;
     memset(&a, 0, sizeof(a));
     a.p = p;
+    a.accept = accept;
+    a.k = k;
+    a.has_h0 = p.h0 != nullptr;
     a.has_gate = p.z != nullptr;
     a.ntiles_d = (int)((p.d_inner + kStepCh - 1) / kStepCh);
     a.ntiles = a.ntiles_d * (int)((p.batch + kStepRows - 1) / kStepRows);
@@ -246,7 +283,20 @@ cudaError_t launch_step_typed(const ScanParams &p, cudaStream_t s) {
     const uint64_t bdims[2] = {kDState, (uint64_t)p.batch};
     const uint64_t bstr[1] = {(uint64_t)kDState * es};
     const uint32_t bbox[2] = {kDState, kStepRows};
-    if (!encode_tmap(&a.tm_state, p.h_out, 4, 3, sdims, sstr, sbox) ||
+    bool ok_maps = true;
+    if constexpr (kResume) {
+        // one row per load: h0 [batch, D, 16] and h_all [batch, k, D, 16]
+        const uint32_t rbox[3] = {kDState, kStepCh, 1};
+        const uint64_t hdims[4] = {kDState, (uint64_t)p.d_inner, (uint64_t)k, (uint64_t)p.batch};
+        const uint64_t hstr[3] = {kDState * 4, (uint64_t)p.d_inner * kDState * 4,
+                                  (uint64_t)k * p.d_inner * kDState * 4};
+        const uint32_t hbox[4] = {kDState, kStepCh, 1, 1};
+        ok_maps = (!p.h0 || encode_tmap(&a.tm_state, p.h0, 4, 3, sdims, sstr, rbox)) &&
+                  encode_tmap(&a.tm_hall, h_all, 4, 4, hdims, hstr, hbox);
+    } else {
+        ok_maps = encode_tmap(&a.tm_state, p.h_out, 4, 3, sdims, sstr, sbox);
+    }
+    if (!ok_maps ||
         !encode_tmap(&a.tm_x, p.x, es, 2, tdims, tstr, tbox) ||
         !encode_tmap(&a.tm_dt, p.dt, es, 2, tdims, tstr, tbox) ||
         (p.z && !encode_tmap(&a.tm_z, p.z, es, 2, tdims, tstr, tbox)) ||
@@ -254,20 +304,20 @@ cudaError_t launch_step_typed(const ScanParams &p, cudaStream_t s) {
         !encode_tmap(&a.tm_C, p.C, es, 2, bdims, bstr, bbox))
         return cudaErrorInvalidValue;
     const size_t smem = sizeof(StepSmem<T>) + 128;
-    auto k = step_kernel<T>;
-    static int ctas = 0;   // resident CTAs per SM x SMs, computed once per process
+    auto kern = step_kernel<T, kResume>;
+    static int ctas = 0;   // resident CTAs per SM x SMs, computed once per process (per instantiation)
     if (ctas == 0) {
-        cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         int dev = 0, sms = 0, per = 0;
         if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
         if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k, kStepThreads, smem)) != cudaSuccess)
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, kern, kStepThreads, smem)) != cudaSuccess)
             return e;
         ctas = sms * (per > 0 ? per : 1);
     }
     const int grid = a.ntiles < ctas ? a.ntiles : ctas;
-    k<<<grid, kStepThreads, smem, s>>>(a);
+    kern<<<grid, kStepThreads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -275,7 +325,15 @@ cudaError_t launch_step_typed(const ScanParams &p, cudaStream_t s) {
 
 cudaError_t launch_step(const ScanParams &p, bool bf16, cudaStream_t s) {
     if (p.batch == 0 || p.d_inner == 0) return cudaSuccess;
-    return bf16 ? launch_step_typed<__nv_bfloat16>(p, s) : launch_step_typed<float>(p, s);
+    return bf16 ? launch_step_typed<__nv_bfloat16, false>(p, nullptr, nullptr, 0, s)
+                : launch_step_typed<float, false>(p, nullptr, nullptr, 0, s);
+}
+
+cudaError_t launch_step_resume(const ScanParams &p, bool bf16, const float *h_all,
+                               const int32_t *accept, int64_t k, cudaStream_t s) {
+    if (p.batch == 0 || p.d_inner == 0) return cudaSuccess;
+    return bf16 ? launch_step_typed<__nv_bfloat16, true>(p, h_all, accept, k, s)
+                : launch_step_typed<float, true>(p, h_all, accept, k, s);
 }
 
 cudaError_t launch_rollback(const float *h0, const float *h_all, const int32_t *accept,

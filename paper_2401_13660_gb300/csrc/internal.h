@@ -38,6 +38,11 @@ bool encode_tmap(CUtensorMap *m, const void *base, int elem_bytes, int rank, con
 cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s);
 cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s);
 cudaError_t launch_step(const ScanParams &p, bool bf16, cudaStream_t s);
+// One step from the state kept after accept[s] drafted bytes: p.h0 (may be
+// null = zeros) when accept[s] == 0, else h_all[s, accept[s]-1]; the new state
+// goes to p.h_out (may alias p.h0).
+cudaError_t launch_step_resume(const ScanParams &p, bool bf16, const float *h_all,
+                               const int32_t *accept, int64_t k, cudaStream_t s);
 cudaError_t launch_accept(const void *logits, bool bf16, const uint8_t *drafted, int64_t streams,
                           int64_t k, int beta, int32_t *accept, cudaStream_t s);
 cudaError_t launch_rollback(const float *h0, const float *h_all, const int32_t *accept,

@@ -199,6 +199,40 @@ mb_status mb_step(const mb_scan_args *args, float *state, void *stream) {
     return from_cuda(mbscan::launch_step(p, args->dtype == MB_BF16, (cudaStream_t)stream));
 }
 
+mb_status mb_step_resume(const mb_scan_args *args, const float *h_all, const int32_t *accept,
+                         int64_t k, float *state, void *ws, size_t ws_bytes, void *stream) {
+    mb_status st = check_args(args, true);
+    if (st != MB_OK) return st;
+    const int64_t chans = args->batch * args->d_inner;
+    if (k < 1 || k > kMaxTokens) return MB_ERR_INVALID_ARG;
+    if (chans > 0 && k > kMaxTokens * 16 / (chans * args->d_state)) return MB_ERR_INVALID_ARG;
+    if (chans == 0) return MB_OK;
+    if (!state || !aligned16(state) || !h_all || !aligned16(h_all) || !accept ||
+        (reinterpret_cast<uintptr_t>(accept) & 3u))
+        return MB_ERR_INVALID_ARG;
+    if (ws && ((reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < mb_workspace_size(args)))
+        return MB_ERR_INVALID_ARG;
+    const int64_t per = args->d_inner * args->d_state * 4;
+    const Range rs = range_of(state, args->batch * per);
+    const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
+    const int64_t tok = chans * es;
+    const Range others[] = {range_of(args->y, tok), range_of(args->x, tok), range_of(args->z, tok),
+                            range_of(args->dt, tok), range_of(args->B, args->batch * args->d_state * es),
+                            range_of(args->C, args->batch * args->d_state * es),
+                            range_of(args->A, args->d_inner * args->d_state * 4),
+                            range_of(h_all, args->batch * k * per), range_of(accept, args->batch * 4)};
+    for (const Range &r : others)
+        if (overlap(rs, r)) return MB_ERR_INVALID_ARG;
+    if (args->h0 && args->h0 != state && overlap(rs, range_of(args->h0, args->batch * per)))
+        return MB_ERR_INVALID_ARG;
+    if (overlap(range_of(args->y, tok), range_of(h_all, args->batch * k * per)) ||
+        overlap(range_of(args->y, tok), range_of(args->h0, args->batch * per)))
+        return MB_ERR_INVALID_ARG;
+    ScanParams p = to_params(args, state, static_cast<StatusBlock *>(ws));
+    return from_cuda(mbscan::launch_step_resume(p, args->dtype == MB_BF16, h_all, accept, k,
+                                                (cudaStream_t)stream));
+}
+
 mb_status mb_check(void *ws, void *stream, int64_t *detail) {
     if (detail) *detail = -1;
     if (ws == nullptr) return MB_ERR_INVALID_ARG;

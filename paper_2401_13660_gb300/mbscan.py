@@ -66,8 +66,9 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
             lib.mb_step.argtypes = [ap, vp, vp]
             lib.mb_check.argtypes = [vp, vp, ctypes.POINTER(i64)]
             lib.mb_accept_topk.argtypes = [vp, ctypes.c_int32, vp, i64, i64, ctypes.c_int32, vp, vp]
+            lib.mb_step_resume.argtypes = [ap, vp, vp, i64, vp, vp, sz, vp]
             for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_check",
-                      "mb_accept_topk"):
+                      "mb_accept_topk", "mb_step_resume"):
                 getattr(lib, f).restype = ctypes.c_int
             lib.mb_status_string.argtypes = [ctypes.c_int]
             lib.mb_status_string.restype = ctypes.c_char_p
@@ -197,6 +198,26 @@ def mb_step(x, dt, B, C, A, y, state, *, z=None, D=None, dt_bias=None, stream=No
     _need(state, "state", torch.float32, (a.batch, a.d_inner, a.d_state), x.device)
     rc = load_library().mb_step(ctypes.byref(a), _ptr(state), _stream(stream))
     _check(rc, "mb_step")
+    return y, state
+
+
+def mb_step_resume(x, dt, B, C, A, y, h_all, accept, state, *, z=None, D=None, dt_bias=None, h0=None,
+                   ws=None, stream=None):
+    """One decode step from the state kept after accept[s] drafted bytes:
+    h0[s] (zeros if None) when accept[s] == 0, else h_all[s, accept[s]-1].
+    x, dt, z, y [batch, 1, d_inner]; B, C [batch, 1, d_state]; h_all [batch,
+    k, d_inner, d_state]; accept [batch] int32; state [batch, d_inner,
+    d_state] is written (it may be h0 itself)."""
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0)
+    _need(h_all, "h_all", torch.float32, None, x.device)
+    if h_all.dim() != 4 or h_all.shape[0] != a.batch or tuple(h_all.shape[2:]) != (a.d_inner, a.d_state):
+        raise ValueError(f"h_all: shape {tuple(h_all.shape)}, expected [batch, k, d_inner, d_state]")
+    _need(accept, "accept", torch.int32, (a.batch,), x.device)
+    _need(state, "state", torch.float32, (a.batch, a.d_inner, a.d_state), x.device)
+    nbytes = 0 if ws is None else ws.numel()
+    rc = load_library().mb_step_resume(ctypes.byref(a), _ptr(h_all), _ptr(accept), h_all.shape[1],
+                                       _ptr(state), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "mb_step_resume")
     return y, state
 
 

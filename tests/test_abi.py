@@ -137,6 +137,27 @@ def test_rollback_checks():
     assert lib.mb_rollback(h0, h_all, acc, out, -1, 16, 64, 16, None, None) == mb.MB_ERR_INVALID_ARG
 
 
+def test_step_resume_checks():
+    lib = mb.load_library()
+    s = _args(L=1)
+    h_all, acc, st, ws = FAKE + (20 << 32), FAKE + (24 << 32), FAKE + (28 << 32), FAKE + (32 << 32)
+
+    def call(a=s, h=h_all, c=acc, k=16, out=st, w=ws, wb=256):
+        return lib.mb_step_resume(ctypes.byref(a), h, c, k, out, w, wb, None)
+
+    assert call(k=0) == mb.MB_ERR_INVALID_ARG                  # k >= 1
+    assert call(h=None) == mb.MB_ERR_INVALID_ARG
+    assert call(c=None) == mb.MB_ERR_INVALID_ARG
+    assert call(c=acc + 2) == mb.MB_ERR_INVALID_ARG            # accept misaligned
+    assert call(out=h_all + 64) == mb.MB_ERR_INVALID_ARG       # state inside h_all
+    assert call(out=s.x) == mb.MB_ERR_INVALID_ARG              # state aliases x
+    assert call(out=s.h0 + 64) == mb.MB_ERR_INVALID_ARG        # partial overlap with h0
+    assert call(wb=16) == mb.MB_ERR_INVALID_ARG                # workspace too small
+    assert call(a=_args(L=2)) == mb.MB_ERR_INVALID_ARG         # seqlen != 1
+    assert call(a=_args(L=1, N=8)) == mb.MB_ERR_UNSUPPORTED
+    assert call(a=_args(batch=0, L=1)) == mb.MB_OK             # nothing to do
+
+
 def test_binding_rejects_cpu_shape_errors():
     import torch
     x = torch.zeros(1, 4, 8, dtype=torch.bfloat16)
