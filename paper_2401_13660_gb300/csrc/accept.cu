@@ -7,12 +7,17 @@
 // rank; a NaN logit is never larger). Drafted byte i is accepted when
 // rank <= beta; a[s] = the first i (0-based) that is not accepted, else k.
 //
-// One warp per stream; lane l compares the 8 logits 8l .. 8l+7 of a position
-// with the drafted byte's logit and the warp sums the counts.
+// One CTA per stream, one warp per drafted position: warp w decides
+// positions w, w + kAccWarps, ... (lane l compares the 8 logits 8l .. 8l+7
+// with the drafted byte's logit, the warp sums the counts); the CTA then takes
+// the first rejected position. Positions are decided kAccWarps at a time, and
+// later groups are skipped once a rejection is found.
 #include "common.cuh"
 
 namespace mbscan {
 namespace {
+
+constexpr int kAccWarps = 16;
 
 __device__ __forceinline__ void load8(const float *p, float (&v)[8]) {
     const float4 a = __ldg(reinterpret_cast<const float4 *>(p));
@@ -30,30 +35,35 @@ __device__ __forceinline__ void load8(const __nv_bfloat16 *p, float (&v)[8]) {
 }
 
 template <typename T>
-__global__ void __launch_bounds__(128) accept_kernel(const T *__restrict__ logits,
-                                                     const uint8_t *__restrict__ drafted,
-                                                     int64_t streams, int64_t k, int beta,
-                                                     int32_t *__restrict__ accept) {
-    const int lane = threadIdx.x & 31;
-    const int64_t s = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
-    if (s >= streams) return;   // whole warp leaves together
-    int a = (int)k;
-    for (int64_t i = 0; i < k; ++i) {
-        const T *row = logits + (s * k + i) * 256;
-        const int byte = __ldg(drafted + s * k + i);
-        const float target = to_f32(row[byte]);
-        float v[8];
-        load8(row + 8 * lane, v);
-        int greater = 0;
+__global__ void __launch_bounds__(32 * kAccWarps) accept_kernel(const T *__restrict__ logits,
+                                                                const uint8_t *__restrict__ drafted,
+                                                                int64_t k, int beta,
+                                                                int32_t *__restrict__ accept) {
+    __shared__ int first_reject;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t s = blockIdx.x;
+    if (threadIdx.x == 0) first_reject = (int)k;
+    __syncthreads();
+    for (int64_t base = 0; base < k; base += kAccWarps) {
+        const int64_t i = base + warp;
+        if (i < k) {
+            const T *row = logits + (s * k + i) * 256;
+            const int byte = __ldg(drafted + s * k + i);
+            const float target = to_f32(row[byte]);
+            float v[8];
+            load8(row + 8 * lane, v);
+            int greater = 0;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) greater += v[j] > target ? 1 : 0;
-        const int rank = 1 + __reduce_add_sync(kFull, greater);
-        if (rank > beta) {   // warp-uniform
-            a = (int)i;
-            break;
+            for (int j = 0; j < 8; ++j) greater += v[j] > target ? 1 : 0;
+            const int rank = 1 + __reduce_add_sync(kFull, greater);
+            if (rank > beta && lane == 0) atomicMin(&first_reject, (int)i);
         }
+        __syncthreads();
+        const bool done = first_reject < (int)k;
+        __syncthreads();   // every thread has read it before the next group can lower it
+        if (done) break;   // uniform
     }
-    if (lane == 0) accept[s] = a;
+    if (threadIdx.x == 0) accept[s] = first_reject;
 }
 
 }  // namespace
@@ -61,13 +71,13 @@ __global__ void __launch_bounds__(128) accept_kernel(const T *__restrict__ logit
 cudaError_t launch_accept(const void *logits, bool bf16, const uint8_t *drafted, int64_t streams,
                           int64_t k, int beta, int32_t *accept, cudaStream_t s) {
     if (streams == 0) return cudaSuccess;
-    const unsigned grid = (unsigned)((streams + 3) / 4);
+    const unsigned grid = (unsigned)streams;
     if (bf16)
-        accept_kernel<__nv_bfloat16><<<grid, 128, 0, s>>>(
-            static_cast<const __nv_bfloat16 *>(logits), drafted, streams, k, beta, accept);
+        accept_kernel<__nv_bfloat16><<<grid, 32 * kAccWarps, 0, s>>>(
+            static_cast<const __nv_bfloat16 *>(logits), drafted, k, beta, accept);
     else
-        accept_kernel<float><<<grid, 128, 0, s>>>(static_cast<const float *>(logits), drafted,
-                                                  streams, k, beta, accept);
+        accept_kernel<float><<<grid, 32 * kAccWarps, 0, s>>>(static_cast<const float *>(logits), drafted,
+                                                             k, beta, accept);
     return cudaGetLastError();
 }
 
