@@ -14,6 +14,8 @@ Functions (MambaByte, Eq. 2-3, discretisation appendix, Table 6, Algorithm 1):
 * ``rollback`` - keep the state after ``accept`` drafted bytes.
 * ``accept_topk`` - Algorithm 1's bifurcation: leading drafted bytes whose
                  rank in the verifier's distribution is within top-beta.
+* ``scan_backward`` - every input gradient of J given dJ/dout and dJ/dh_last
+                 (the training path), by the adjoint recurrence in fp64.
 
 Inputs are widened exactly to float64 before the call (bf16 and fp32 values
 are exactly representable in fp64).
@@ -64,6 +66,8 @@ def _load():
             lib.oracle_rollback.argtypes = [i64, i64, i64, i64, dp, dp,
                                             ctypes.POINTER(ctypes.c_int32), dp]
             lib.oracle_rollback.restype = ctypes.c_int
+            lib.oracle_scan_backward.argtypes = [i64, i64, i64, i64] + [dp] * 11 + [dp] * 9 + [ctypes.c_int]
+            lib.oracle_scan_backward.restype = ctypes.c_int
             _lib = lib
     return _lib
 
@@ -108,6 +112,36 @@ def scan(x, dt, B, C, A, *, z=None, D=None, dt_bias=None, h0=None, b_rule=B_EULE
     if rc != 0:
         raise RuntimeError(f"oracle_scan failed ({rc})")
     return y, h_last, h_all
+
+
+def scan_backward(x, dt, B, C, A, dout, *, z=None, D=None, dt_bias=None, h0=None, dh_last=None,
+                  nthreads=None):
+    """Gradients of J, given dJ/dout [batch, L, D] and dJ/dh_last [batch, D, N]
+    (None = 0), for the Euler-rule layer core. Returns a dict with dx, dz
+    (None without a gate), ddt [batch, L, D]; dB, dC [batch, L, N]; dA [D, N];
+    dD, ddt_bias [D]; dh0 [batch, D, N] (all float64)."""
+    x, dt, B, C, A, dout = map(_f64, (x, dt, B, C, A, dout))
+    z, D, dt_bias, h0, dh_last = map(_f64, (z, D, dt_bias, h0, dh_last))
+    batch, L, Dn = x.shape
+    N = A.shape[1]
+    assert dt.shape == x.shape and dout.shape == x.shape
+    assert B.shape == (batch, L, N) and C.shape == (batch, L, N) and A.shape == (Dn, N)
+    g = {k: np.empty((batch, L, Dn)) for k in ("dx", "ddt")}
+    g["dz"] = np.empty((batch, L, Dn)) if z is not None else None
+    g["dB"] = np.empty((batch, L, N))
+    g["dC"] = np.empty((batch, L, N))
+    g["dA"] = np.empty((Dn, N))
+    g["dD"] = np.empty(Dn)
+    g["ddt_bias"] = np.empty(Dn)
+    g["dh0"] = np.empty((batch, Dn, N))
+    rc = _load().oracle_scan_backward(
+        batch, L, Dn, N, _ptr(x), _ptr(z), _ptr(dt), _ptr(B), _ptr(C), _ptr(A), _ptr(D), _ptr(dt_bias),
+        _ptr(h0), _ptr(dout), _ptr(dh_last), _ptr(g["dx"]), _ptr(g["dz"]), _ptr(g["ddt"]), _ptr(g["dB"]),
+        _ptr(g["dC"]), _ptr(g["dA"]), _ptr(g["dD"]), _ptr(g["ddt_bias"]), _ptr(g["dh0"]),
+        int(nthreads or default_threads()))
+    if rc != 0:
+        raise RuntimeError(f"oracle_scan_backward failed ({rc})")
+    return g
 
 
 def step(state, x, dt, B, C, A, *, z=None, D=None, dt_bias=None, b_rule=B_EULER, nthreads=None):
