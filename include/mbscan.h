@@ -175,6 +175,58 @@ mb_status mb_step(const mb_scan_args *args, float *state, void *stream);
 mb_status mb_step_resume(const mb_scan_args *args, const float *h_all, const int32_t *accept,
                          int64_t k, float *state, void *ws, size_t ws_bytes, void *stream);
 
+/* ------------------------------------------------------------------------
+ * Training path (the paper trains through this scan: Section 2 "parallel
+ * scans", Section 4 training setup, L = 8192, bf16 mixed precision).
+ * ------------------------------------------------------------------------ */
+
+/* Steps between the state checkpoints that the training forward keeps for
+ * the backward (the backward recomputes the states inside each chunk). */
+#define MB_CKPT_STEPS 16
+
+/*
+ * Training forward: mb_scan_prefill that also writes the state before every
+ * MB_CKPT_STEPS-step chunk:
+ *   h_ckpt[b, i, d, n] = state before step i * MB_CKPT_STEPS, fp32, shape
+ *   [batch, ceil(seqlen / MB_CKPT_STEPS), d_inner, d_state] (h_ckpt[b, 0] is
+ *   h0, or zeros). Everything else is as for mb_scan_prefill. h_ckpt must
+ *   not overlap any other argument.
+ */
+mb_status mb_scan_prefill_ckpt(const mb_scan_args *args, float *h_last, float *h_ckpt, void *ws,
+                               size_t ws_bytes, void *stream);
+
+/* Gradients written by mb_scan_backward (device pointers, overwritten). */
+typedef struct {
+    void *dx, *dz, *ddt;   /* [batch, seqlen, d_inner], dtype; dz is required when args->z is
+                              not NULL and ignored otherwise */
+    float *dB, *dC;        /* [batch, seqlen, d_state] fp32 (sums over channels) */
+    float *dA;             /* [d_inner, d_state] fp32 */
+    float *dD, *ddt_bias;  /* [d_inner] fp32, or NULL to skip */
+    float *dh0;            /* [batch, d_inner, d_state] fp32 (dJ/dh0), or NULL to skip */
+} mb_scan_grads;
+
+/*
+ * Backward of the layer core: every input gradient of a scalar J given
+ *   dout    : dJ/dy [batch, seqlen, d_inner], dtype (y as written by the
+ *             forward, i.e. after the gate)
+ *   dh_last : dJ/dh_last [batch, d_inner, d_state] fp32, or NULL (= 0)
+ * args: the forward's arguments (args->y is not read and may be NULL);
+ * h_ckpt: the checkpoints written by mb_scan_prefill_ckpt for the same args.
+ * The adjoint recurrence (Eq. 2 transposed), per (b, d) from t = L-1 down to
+ * 0 with g = dJ/dh_t:
+ *   dy = dout * silu(z), dz = dout * y_t * silu'(z), g += dy C_t,
+ *   dC_t += dy h_t, dx_t = dy D + Delta_t g.B_t, dB_t += g Delta_t x_t,
+ *   dDelta_t = x_t g.B_t + sum_n g Abar h_{t-1} A, dA += g Abar h_{t-1} Delta_t,
+ *   g = Abar g, ddt_t = dDelta_t sigmoid(dt_t + dt_bias), dD += dy x_t,
+ *   dt_bias gradient = sum of ddt; dh0 = g after t = 0.
+ * Sums over channels (dB, dC) and over batch rows (dA, dD, ddt_bias) are
+ * accumulated with fp32 atomics: their rounding order is not fixed. The
+ * outputs must not overlap the inputs or each other. ws as for prefill.
+ */
+mb_status mb_scan_backward(const mb_scan_args *args, const float *h_ckpt, const void *dout,
+                           const float *dh_last, const mb_scan_grads *grads, void *ws,
+                           size_t ws_bytes, void *stream);
+
 /*
  * Read and clear the status block of a workspace (blocking: waits for
  * `stream`). Returns MB_OK, or the first device-side error recorded by

@@ -24,9 +24,11 @@ struct ScanParams {
     void *y;
     float *h_out;      // prefill: h_last (may be null); verify: h_all; step: state
     StatusBlock *status;
+    float *h_ckpt;     // prefill with checkpoints: state before every kCkptSteps-step chunk
 };
 
 constexpr int kDState = 16;
+constexpr int kCkptSteps = 16;   // steps between the state checkpoints of the training forward
 
 // Encode a tiled TMA tensor map over `base` (bf16 when elem_bytes == 2, else
 // fp32): dims innermost first, strides[i] = byte stride of dimension i + 1,
@@ -37,6 +39,20 @@ bool encode_tmap(CUtensorMap *m, const void *base, int elem_bytes, int rank, con
 // Launchers: return the cudaError_t of the launch.
 cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s);
 cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s);
+// Prefill that also writes p.h_ckpt [batch, ceil(L / kCkptSteps), d_inner, 16].
+cudaError_t launch_prefill_ckpt(const ScanParams &p, bool bf16, cudaStream_t s);
+// Backward of the layer core (backward.cu).
+struct GradParams {
+    const float *h_ckpt;          // [batch, nchunks, d_inner, 16] from launch_prefill_ckpt
+    const void *dout;             // [batch, L, d_inner], input dtype
+    const float *dh_last;         // [batch, d_inner, 16] or null
+    void *dx, *dz, *ddt;          // [batch, L, d_inner], input dtype (dz null without a gate)
+    float *dB, *dC;               // [batch, L, 16]
+    float *dA;                    // [d_inner, 16]
+    float *dD, *ddt_bias;         // [d_inner] or null
+    float *dh0;                   // [batch, d_inner, 16] or null
+};
+cudaError_t launch_backward(const ScanParams &p, const GradParams &g, bool bf16, cudaStream_t s);
 cudaError_t launch_step(const ScanParams &p, bool bf16, cudaStream_t s);
 // One step from the state kept after accept[s] drafted bytes: p.h0 (may be
 // null = zeros) when accept[s] == 0, else h_all[s, accept[s]-1]; the new state

@@ -20,9 +20,9 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 struct Range {
     uintptr_t lo, hi;
 };
-Range range_of(const void *p, int64_t bytes) {
+Range range_of(const void *p, int64_t bytes) {   // a null pointer is an empty range
     uintptr_t a = reinterpret_cast<uintptr_t>(p);
-    return Range{a, a + (uintptr_t)(bytes > 0 ? bytes : 0)};
+    return Range{a, p ? a + (uintptr_t)(bytes > 0 ? bytes : 0) : a};
 }
 bool overlap(Range a, Range b) { return a.lo < b.hi && b.lo < a.hi && a.lo != a.hi && b.lo != b.hi; }
 
@@ -31,7 +31,7 @@ bool overlap(Range a, Range b) { return a.lo < b.hi && b.lo < a.hi && a.lo != a.
 constexpr int64_t kMaxTokens = (int64_t)1 << 31;
 
 // Validate the common part of a scan problem; `need_seqlen1` for mb_step.
-mb_status check_args(const mb_scan_args *a, bool need_seqlen1) {
+mb_status check_args(const mb_scan_args *a, bool need_seqlen1, bool need_y = true) {
     if (a == nullptr) return MB_ERR_INVALID_ARG;
     if (a->batch < 0 || a->seqlen < 0 || a->d_inner < 0 || a->d_state < 0) return MB_ERR_INVALID_ARG;
     if (a->dtype != MB_F32 && a->dtype != MB_BF16) return MB_ERR_INVALID_ARG;
@@ -45,7 +45,7 @@ mb_status check_args(const mb_scan_args *a, bool need_seqlen1) {
     if (chans > kMaxTokens / mbscan::kDState) return MB_ERR_INVALID_ARG;
     const bool any_tokens = a->batch * a->seqlen * a->d_inner > 0;
     const bool any_chan = chans > 0;
-    if (any_tokens && (!a->x || !a->dt || !a->B || !a->C || !a->y)) return MB_ERR_INVALID_ARG;
+    if (any_tokens && (!a->x || !a->dt || !a->B || !a->C || (need_y && !a->y))) return MB_ERR_INVALID_ARG;
     if (any_chan && !a->A) return MB_ERR_INVALID_ARG;
     const void *ptrs[] = {a->x, a->z, a->dt, a->B, a->C, a->A, a->D, a->dt_bias, a->h0, a->y};
     for (const void *p : ptrs)
@@ -75,6 +75,7 @@ ScanParams to_params(const mb_scan_args *a, float *h_out, StatusBlock *status) {
     p.y = a->y;
     p.h_out = h_out;
     p.status = status;
+    p.h_ckpt = nullptr;
     return p;
 }
 
@@ -93,7 +94,7 @@ mb_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MB_OK : MB_ERR_CU
 extern "C" {
 
 size_t mb_workspace_size(const mb_scan_args *args) {
-    if (check_args(args, false) != MB_OK) return 0;
+    if (check_args(args, false, false) != MB_OK) return 0;
     return mbscan::kStatusBytes;
 }
 
@@ -231,6 +232,92 @@ mb_status mb_step_resume(const mb_scan_args *args, const float *h_all, const int
     ScanParams p = to_params(args, state, static_cast<StatusBlock *>(ws));
     return from_cuda(mbscan::launch_step_resume(p, args->dtype == MB_BF16, h_all, accept, k,
                                                 (cudaStream_t)stream));
+}
+
+mb_status mb_scan_prefill_ckpt(const mb_scan_args *args, float *h_last, float *h_ckpt, void *ws,
+                               size_t ws_bytes, void *stream) {
+    mb_status st = check_args(args, false);
+    if (st != MB_OK) return st;
+    if ((st = check_ws(args, ws, ws_bytes)) != MB_OK) return st;
+    const int64_t chans = args->batch * args->d_inner;
+    const int64_t nchunks = (args->seqlen + mbscan::kCkptSteps - 1) / mbscan::kCkptSteps;
+    const int64_t ck_bytes = chans * nchunks * args->d_state * 4;
+    if (chans > 0 && nchunks > 0 && (!h_ckpt || !aligned16(h_ckpt))) return MB_ERR_INVALID_ARG;
+    if (h_last && !aligned16(h_last)) return MB_ERR_INVALID_ARG;
+    const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
+    const int64_t tok = chans * args->seqlen * es;
+    const int64_t bc = args->batch * args->seqlen * args->d_state * es;
+    const Range rc = range_of(h_ckpt, ck_bytes);
+    const Range others[] = {range_of(args->x, tok), range_of(args->z, tok), range_of(args->dt, tok),
+                            range_of(args->B, bc), range_of(args->C, bc), range_of(args->y, tok),
+                            range_of(args->A, args->d_inner * args->d_state * 4),
+                            range_of(args->h0, chans * args->d_state * 4),
+                            range_of(h_last, chans * args->d_state * 4), range_of(ws, ws_bytes)};
+    for (const Range &r : others)
+        if (overlap(rc, r)) return MB_ERR_INVALID_ARG;
+    if (h_last && h_last != args->h0 && overlap(range_of(h_last, chans * args->d_state * 4),
+                                                range_of(args->h0, chans * args->d_state * 4)))
+        return MB_ERR_INVALID_ARG;
+    ScanParams p = to_params(args, h_last, static_cast<StatusBlock *>(ws));
+    p.h_ckpt = h_ckpt;
+    return from_cuda(mbscan::launch_prefill_ckpt(p, args->dtype == MB_BF16, (cudaStream_t)stream));
+}
+
+mb_status mb_scan_backward(const mb_scan_args *args, const float *h_ckpt, const void *dout,
+                           const float *dh_last, const mb_scan_grads *grads, void *ws,
+                           size_t ws_bytes, void *stream) {
+    mb_status st = check_args(args, false, false);
+    if (st != MB_OK) return st;
+    if (!grads) return MB_ERR_INVALID_ARG;
+    if ((st = check_ws(args, ws, ws_bytes)) != MB_OK) return st;
+    const int64_t Bn = args->batch, L = args->seqlen, Dn = args->d_inner, N = args->d_state;
+    const int64_t chans = Bn * Dn;
+    const bool any_tokens = chans * L > 0;
+    const mb_scan_grads &g = *grads;
+    if (Dn > 0 && (!g.dA || !aligned16(g.dA))) return MB_ERR_INVALID_ARG;
+    if (Bn * L > 0 && (!g.dB || !g.dC || !aligned16(g.dB) || !aligned16(g.dC))) return MB_ERR_INVALID_ARG;
+    if (any_tokens && (!h_ckpt || !dout || !g.dx || !g.ddt || (args->z && !g.dz)))
+        return MB_ERR_INVALID_ARG;
+    const void *al[] = {h_ckpt, dout, dh_last, g.dx, g.ddt, args->z ? g.dz : nullptr, g.dD, g.ddt_bias,
+                        g.dh0};
+    for (const void *q : al)
+        if (q && !aligned16(q)) return MB_ERR_INVALID_ARG;
+    const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
+    const int64_t tok = chans * L * es, bcb = Bn * L * N * es, st_b = chans * N * 4;
+    const int64_t nchunks = (L + mbscan::kCkptSteps - 1) / mbscan::kCkptSteps;
+    // outputs: disjoint from each other and from every input
+    const Range outs[] = {range_of(g.dx, any_tokens ? tok : 0), range_of(g.ddt, any_tokens ? tok : 0),
+                          range_of(args->z ? g.dz : nullptr, any_tokens ? tok : 0),
+                          range_of(g.dB, Bn * L * N * 4), range_of(g.dC, Bn * L * N * 4),
+                          range_of(g.dA, Dn * N * 4), range_of(g.dD, Dn * 4), range_of(g.ddt_bias, Dn * 4),
+                          range_of(g.dh0, st_b)};
+    const Range ins[] = {range_of(args->x, tok), range_of(args->z, tok), range_of(args->dt, tok),
+                         range_of(args->B, bcb), range_of(args->C, bcb), range_of(args->A, Dn * N * 4),
+                         range_of(args->D, Dn * 4), range_of(args->dt_bias, Dn * 4), range_of(args->h0, st_b),
+                         range_of(h_ckpt, chans * nchunks * N * 4), range_of(dout, tok),
+                         range_of(dh_last, st_b), range_of(ws, ws_bytes)};
+    constexpr int kOuts = sizeof(outs) / sizeof(outs[0]);
+    for (int i = 0; i < kOuts; ++i) {
+        for (const Range &r : ins)
+            if (overlap(outs[i], r)) return MB_ERR_INVALID_ARG;
+        for (int j = i + 1; j < kOuts; ++j)
+            if (overlap(outs[i], outs[j])) return MB_ERR_INVALID_ARG;
+    }
+    ScanParams p = to_params(args, nullptr, static_cast<StatusBlock *>(ws));
+    mbscan::GradParams gp;
+    gp.h_ckpt = h_ckpt;
+    gp.dout = dout;
+    gp.dh_last = dh_last;
+    gp.dx = g.dx;
+    gp.dz = args->z ? g.dz : nullptr;
+    gp.ddt = g.ddt;
+    gp.dB = g.dB;
+    gp.dC = g.dC;
+    gp.dA = g.dA;
+    gp.dD = g.dD;
+    gp.ddt_bias = g.ddt_bias;
+    gp.dh0 = g.dh0;
+    return from_cuda(mbscan::launch_backward(p, gp, args->dtype == MB_BF16, (cudaStream_t)stream));
 }
 
 mb_status mb_check(void *ws, void *stream, int64_t *detail) {

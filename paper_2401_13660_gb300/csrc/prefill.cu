@@ -187,7 +187,7 @@ __device__ __forceinline__ float reduce_steps(const float (&part)[LPC], int q) {
     }
 }
 
-template <typename T, int LPC, int STAGES, bool kStoreAll>
+template <typename T, int LPC, int STAGES, bool kStoreAll, bool kCkpt>
 __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant__ PrefillArgs a) {
     using G = Geom<LPC>;
     constexpr int CH = G::kCh;
@@ -266,6 +266,16 @@ __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant
         if (has_next && ok) convert(s.cv[(i + 1) & 1], s.raw[nst], cr, t0 + kT, L, gate);
 
         // (2) chunk i: decays of all kT steps, recurrence, shares of C.h
+        if constexpr (kCkpt) {   // state before chunk i, for the backward's recompute
+            static_assert(kT == kCkptSteps, "checkpoints are taken per chunk");
+            if (chan_ok) {
+                float2 *dst = reinterpret_cast<float2 *>(
+                    p.h_ckpt + (((int64_t)b * nchunks + i) * D + d) * kDState + G::kSPL * q);
+#pragma unroll
+                for (int k = 0; k < G::kPairs; k += 2)
+                    *reinterpret_cast<float4 *>(dst + k) = make_float4(h[k].x, h[k].y, h[k + 1].x, h[k + 1].y);
+            }
+        }
         const Conv<CH> &cv = s.cv[i & 1];
         const Raw<T, CH> &rs = s.raw[i % STAGES];   // B, C straight from the TMA tile
         float2 ab[kT][G::kPairs];
@@ -368,7 +378,7 @@ bool make_map(CUtensorMap *m, const void *base, bool bf16, int64_t batch, int64_
     return encode_tmap(m, base, (int)es, 3, dims, strides, box);
 }
 
-template <typename T, int LPC, int STAGES, bool kStoreAll>
+template <typename T, int LPC, int STAGES, bool kStoreAll, bool kCkpt = false>
 cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
     constexpr int kCh = Geom<LPC>::kCh;
     const bool bf16 = sizeof(T) == 2;
@@ -384,7 +394,7 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
         !make_map(&a.tm_y, p.y, bf16, p.batch, p.seqlen, p.d_inner, kCh))
         return cudaErrorInvalidValue;
     const size_t smem = sizeof(Smem<T, kCh, STAGES>) + 128;
-    auto k = prefill_kernel<T, LPC, STAGES, kStoreAll>;
+    auto k = prefill_kernel<T, LPC, STAGES, kStoreAll, kCkpt>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const dim3 grid((unsigned)(((p.d_inner + kCh - 1) / kCh) * p.batch));
@@ -409,6 +419,14 @@ cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s) {
     constexpr int LPC = kPrefillLanesPerChannel;
     return bf16 ? launch_typed<__nv_bfloat16, LPC, kPrefillStages, false>(p, s)
                 : launch_typed<float, LPC, kPrefillStages, false>(p, s);
+}
+
+cudaError_t launch_prefill_ckpt(const ScanParams &p, bool bf16, cudaStream_t s) {
+    if (p.batch == 0 || p.d_inner == 0) return cudaSuccess;
+    if (p.seqlen == 0) return launch_prefill(p, bf16, s);   // no chunks: no checkpoints
+    constexpr int LPC = kPrefillLanesPerChannel;
+    return bf16 ? launch_typed<__nv_bfloat16, LPC, kPrefillStages, false, true>(p, s)
+                : launch_typed<float, LPC, kPrefillStages, false, true>(p, s);
 }
 
 cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s) {

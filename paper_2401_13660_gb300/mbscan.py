@@ -43,6 +43,15 @@ class mb_scan_args(ctypes.Structure):
     ]
 
 
+class mb_scan_grads(ctypes.Structure):
+    _fields_ = [("dx", ctypes.c_void_p), ("dz", ctypes.c_void_p), ("ddt", ctypes.c_void_p),
+                ("dB", ctypes.c_void_p), ("dC", ctypes.c_void_p), ("dA", ctypes.c_void_p),
+                ("dD", ctypes.c_void_p), ("ddt_bias", ctypes.c_void_p), ("dh0", ctypes.c_void_p)]
+
+
+MB_CKPT_STEPS = 16
+
+
 def library_path() -> str:
     return _build.LIB
 
@@ -67,8 +76,10 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
             lib.mb_check.argtypes = [vp, vp, ctypes.POINTER(i64)]
             lib.mb_accept_topk.argtypes = [vp, ctypes.c_int32, vp, i64, i64, ctypes.c_int32, vp, vp]
             lib.mb_step_resume.argtypes = [ap, vp, vp, i64, vp, vp, sz, vp]
+            lib.mb_scan_prefill_ckpt.argtypes = [ap, vp, vp, vp, sz, vp]
+            lib.mb_scan_backward.argtypes = [ap, vp, vp, vp, ctypes.POINTER(mb_scan_grads), vp, sz, vp]
             for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_check",
-                      "mb_accept_topk", "mb_step_resume"):
+                      "mb_accept_topk", "mb_step_resume", "mb_scan_prefill_ckpt", "mb_scan_backward"):
                 getattr(lib, f).restype = ctypes.c_int
             lib.mb_status_string.argtypes = [ctypes.c_int]
             lib.mb_status_string.restype = ctypes.c_char_p
@@ -199,6 +210,65 @@ def mb_step(x, dt, B, C, A, y, state, *, z=None, D=None, dt_bias=None, stream=No
     rc = load_library().mb_step(ctypes.byref(a), _ptr(state), _stream(stream))
     _check(rc, "mb_step")
     return y, state
+
+
+def mb_scan_prefill_ckpt(x, dt, B, C, A, y, h_ckpt=None, *, z=None, D=None, dt_bias=None, h0=None,
+                         h_last=None, ws=None, stream=None):
+    """Training forward: prefill that also writes h_ckpt [batch, ceil(L / 16),
+    d_inner, d_state], the state before every 16-step chunk (allocated when
+    None). Returns (y, h_last, h_ckpt)."""
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0)
+    nch = (a.seqlen + MB_CKPT_STEPS - 1) // MB_CKPT_STEPS
+    if h_ckpt is None:
+        h_ckpt = torch.empty(a.batch, nch, a.d_inner, a.d_state, dtype=torch.float32, device=x.device)
+    _need(h_ckpt, "h_ckpt", torch.float32, (a.batch, nch, a.d_inner, a.d_state), x.device)
+    _need(h_last, "h_last", torch.float32, (a.batch, a.d_inner, a.d_state), x.device)
+    if ws is None:
+        ws = new_workspace(a, x.device)
+    rc = load_library().mb_scan_prefill_ckpt(ctypes.byref(a), _ptr(h_last), _ptr(h_ckpt), _ptr(ws),
+                                             ws.numel(), _stream(stream))
+    _check(rc, "mb_scan_prefill_ckpt")
+    return y, h_last, h_ckpt
+
+
+def mb_scan_backward(x, dt, B, C, A, h_ckpt, dout, *, z=None, D=None, dt_bias=None, h0=None,
+                     dh_last=None, grads=None, ws=None, stream=None):
+    """Backward of the layer core. Returns a dict of gradients: dx, ddt, dz (or
+    None) in the input dtype [batch, L, d_inner]; dB, dC fp32 [batch, L,
+    d_state]; dA fp32 [d_inner, d_state]; dD, ddt_bias fp32 [d_inner]; dh0 fp32
+    [batch, d_inner, d_state]. Tensors missing from `grads` are allocated."""
+    if x.dtype not in _DTYPES:
+        raise TypeError(f"unsupported input dtype {x.dtype}")
+    batch, L, Dn = x.shape
+    N = A.shape[1]
+    dev = x.device
+    a = make_args(x, dt, B, C, A, x, z=z, D=D, dt_bias=dt_bias, h0=h0)
+    a.y = None
+    nch = (L + MB_CKPT_STEPS - 1) // MB_CKPT_STEPS
+    _need(h_ckpt, "h_ckpt", torch.float32, (batch, nch, Dn, N), dev)
+    _need(dout, "dout", x.dtype, (batch, L, Dn), dev)
+    _need(dh_last, "dh_last", torch.float32, (batch, Dn, N), dev)
+    g = dict(grads or {})
+    shapes = {"dx": ((batch, L, Dn), x.dtype), "ddt": ((batch, L, Dn), x.dtype),
+              "dz": ((batch, L, Dn), x.dtype), "dB": ((batch, L, N), torch.float32),
+              "dC": ((batch, L, N), torch.float32), "dA": ((Dn, N), torch.float32),
+              "dD": ((Dn,), torch.float32), "ddt_bias": ((Dn,), torch.float32),
+              "dh0": ((batch, Dn, N), torch.float32)}
+    for k, (shp, dty) in shapes.items():
+        if k == "dz" and z is None:
+            g[k] = None
+            continue
+        if g.get(k) is None:
+            g[k] = torch.empty(shp, dtype=dty, device=dev)
+        _need(g[k], k, dty, shp, dev)
+    st = mb_scan_grads(*(None if g[k] is None else g[k].data_ptr() for k in
+                         ("dx", "dz", "ddt", "dB", "dC", "dA", "dD", "ddt_bias", "dh0")))
+    if ws is None:
+        ws = new_workspace(a, dev)
+    rc = load_library().mb_scan_backward(ctypes.byref(a), _ptr(h_ckpt), _ptr(dout), _ptr(dh_last),
+                                         ctypes.byref(st), _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "mb_scan_backward")
+    return g
 
 
 def mb_step_resume(x, dt, B, C, A, y, h_all, accept, state, *, z=None, D=None, dt_bias=None, h0=None,

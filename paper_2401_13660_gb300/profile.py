@@ -34,12 +34,19 @@ def algorithmic_bytes(entry: str, w, s_in: int) -> int:
         return 2 * b * D * N * 4 + b * 4
     if entry == "step":
         return 2 * b * D * N * 4 + 3 * b * D * s_in + 2 * b * N * s_in + params + b * D * s_in
+    if entry == "backward":
+        nch = (L + 15) // 16
+        rd = 4 * b * L * D * s_in + 2 * b * L * N * s_in + params + b * nch * D * N * 4
+        rd += b * D * N * 4 if w.h0 != "zeros" else 0
+        rd += b * D * N * 4   # dh_last
+        wr = 3 * b * L * D * s_in + 2 * b * L * N * 4 + D * N * 4 + 2 * D * 4 + b * D * N * 4
+        return rd + wr
     raise ValueError(entry)
 
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--entry", choices=["prefill", "verify", "rollback", "step"], required=True)
+    ap.add_argument("--entry", choices=["prefill", "verify", "rollback", "step", "backward"], required=True)
     ap.add_argument("--workload", required=True, choices=sorted(WORKLOADS))
     ap.add_argument("--iters", type=int, default=5)
     ap.add_argument("--layers", type=int, default=4, help="state sets cycled by --entry step")
@@ -56,7 +63,7 @@ def main():
         inp["ws"] = torch.zeros(256, dtype=torch.uint8, device=dev)
         if inp["h0"] is None and a.entry in ("verify", "rollback", "step"):
             inp["h0"] = torch.zeros(w.batch, w.d_inner, N_STATE, device=dev)
-        if a.entry == "prefill":
+        if a.entry in ("prefill", "backward"):
             inp["h_last"] = torch.empty(w.batch, w.d_inner, N_STATE, device=dev)
         if a.entry in ("verify", "rollback"):
             inp["h_all"] = torch.empty(w.batch, w.seqlen, w.d_inner, N_STATE, device=dev)
@@ -69,6 +76,17 @@ def main():
                 inp[k] = inp[k][:, :1].contiguous()
             inp["state"] = inp["h0"].clone()
         sets.append(inp)
+    if a.entry == "backward":   # the training forward provides the checkpoints
+        s0 = sets[0]
+        _, _, s0["h_ckpt"] = mb.mb_scan_prefill_ckpt(s0["x"], s0["dt"], s0["B"], s0["C"], s0["A"], s0["y"],
+                                                     z=s0["z"], D=s0["D"], dt_bias=s0["dt_bias"], h0=s0["h0"],
+                                                     h_last=s0["h_last"], ws=s0["ws"])
+        gen = torch.Generator(device=dev).manual_seed(5)
+        s0["dout"] = torch.randn(s0["x"].shape, device=dev, generator=gen).to(s0["x"].dtype)
+        s0["dh_last"] = torch.randn(s0["h_last"].shape, device=dev, generator=gen)
+        s0["grads"] = mb.mb_scan_backward(s0["x"], s0["dt"], s0["B"], s0["C"], s0["A"], s0["h_ckpt"],
+                                          s0["dout"], z=s0["z"], D=s0["D"], dt_bias=s0["dt_bias"],
+                                          h0=s0["h0"], dh_last=s0["dh_last"], ws=s0["ws"])
     if a.entry == "rollback":
         s0 = sets[0]
         mb.mb_scan_verify(s0["x"], s0["dt"], s0["B"], s0["C"], s0["A"], s0["y"], s0["h_all"],
@@ -86,6 +104,10 @@ def main():
                               D=s["D"], dt_bias=s["dt_bias"], h0=s["h0"], ws=s["ws"], stream=stream)
         elif a.entry == "rollback":
             mb.mb_rollback(s["h0"], s["h_all"], s["accept"], s["h_out"], ws=s["ws"], stream=stream)
+        elif a.entry == "backward":
+            mb.mb_scan_backward(s["x"], s["dt"], s["B"], s["C"], s["A"], s["h_ckpt"], s["dout"], z=s["z"],
+                                D=s["D"], dt_bias=s["dt_bias"], h0=s["h0"], dh_last=s["dh_last"],
+                                grads=s["grads"], ws=s["ws"], stream=stream)
         else:
             mb.mb_step(s["x"], s["dt"], s["B"], s["C"], s["A"], s["y"], s["state"], z=s["z"],
                        D=s["D"], dt_bias=s["dt_bias"], stream=stream)

@@ -158,6 +158,42 @@ def test_step_resume_checks():
     assert call(a=_args(batch=0, L=1)) == mb.MB_OK             # nothing to do
 
 
+def test_training_path_checks():
+    lib = mb.load_library()
+    a = _args(L=40)
+    ck, ws = FAKE + (40 << 32), FAKE + (200 << 32)
+    assert lib.mb_scan_prefill_ckpt(ctypes.byref(a), None, None, ws, 256, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_scan_prefill_ckpt(ctypes.byref(a), None, a.x, ws, 256, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_scan_prefill_ckpt(ctypes.byref(a), None, ck + 8, ws, 256, None) == mb.MB_ERR_INVALID_ARG
+
+    def grads(**kw):
+        base = FAKE + (60 << 32)
+        g = mb.mb_scan_grads(*(base + i * (1 << 32) for i in range(9)))
+        for k, v in kw.items():
+            setattr(g, k, v)
+        return g
+
+    dout = FAKE + (50 << 32)
+
+    def bwd(args=a, h=ck, o=dout, g=None):
+        return lib.mb_scan_backward(ctypes.byref(args), h, o, None, ctypes.byref(g or grads()), ws, 256, None)
+
+    b = _args(L=40, y=None)                                  # y is not needed by the backward
+    assert bwd(args=b, h=None) == mb.MB_ERR_INVALID_ARG      # checkpoints required
+    assert bwd(args=b, o=None) == mb.MB_ERR_INVALID_ARG      # dout required
+    assert bwd(args=b, g=grads(dz=None)) == mb.MB_ERR_INVALID_ARG     # gate present, dz missing
+    assert bwd(args=b, g=grads(dx=b.x)) == mb.MB_ERR_INVALID_ARG      # output aliases an input
+    g2 = grads()
+    g2.ddt = g2.dx + 64
+    assert bwd(args=b, g=g2) == mb.MB_ERR_INVALID_ARG        # outputs overlap
+    assert bwd(args=_args(L=40, N=8)) == mb.MB_ERR_UNSUPPORTED
+    assert lib.mb_scan_backward(ctypes.byref(b), ck, dout, None, None, ws, 256, None) == mb.MB_ERR_INVALID_ARG
+    # optional outputs left out (null) pass validation (the call then fails to launch: no GPU here)
+    nz = _args(L=40, y=None, z=None)
+    want_launch = (mb.MB_OK, mb.MB_ERR_CUDA)
+    assert bwd(args=nz, g=grads(dz=None, dD=None, ddt_bias=None, dh0=None)) in want_launch
+
+
 def test_binding_rejects_cpu_shape_errors():
     import torch
     x = torch.zeros(1, 4, 8, dtype=torch.bfloat16)
