@@ -16,8 +16,8 @@
 // 4q .. 4q+3 of channel warp*8 + c8. Chunks of kCkptSteps steps are taken in
 // reverse order through a ring of 3-D TMA tile loads (dt, x, z, dout, B, C).
 // Per chunk:
-//  * conversion (once per (t, channel pair), for the next chunk): Delta,
-//    Delta*x, x, dy, sigmoid(dt + bias), dout * silu'(z) into shared memory;
+//  * conversion (once per (t, channel pair)): Delta, Delta*x, x, dy into
+//    shared memory;
 //  * recompute: from the chunk's checkpoint, the forward states of the 16
 //    steps (to shared memory, one float4 per lane and step) and each lane's
 //    share of C.h (for y);
@@ -27,8 +27,12 @@
 //    shared memory per warp; S1, S2 and y are summed over the 4 lanes of a
 //    channel with a transposed 2-round reduction per 4 steps, after which lane
 //    q finishes step 4m+q (dx, ddt, dz to output tiles written by TMA stores);
-//  * after the chunk's barrier (in the next iteration), the 4 warps' dB, dC
-//    shares are added and sent to global memory with vector atomics.
+//    The finishing lane evaluates sigmoid(dt + bias) and silu'(z) itself from
+//    the chunk's tiles;
+//  * after the chunk's barrier (in the next iteration), the CTA's dB, dC sums
+//    are sent to global memory with vector atomics.
+// Two barriers per chunk (after the conversion, after the sweep) keep one
+// conversion buffer and one dB/dC buffer, so that 4 CTAs fit on an SM.
 // dA, dD, dbias are accumulated in registers and added atomically at the end
 // (one contribution per batch row); dh0 is stored directly.
 #include <string.h>
@@ -57,16 +61,15 @@ struct BRaw {  // TMA destinations; member offsets are multiples of 128 B
 
 struct BConv {
     float4 a[kBT][kBCh];   // (Delta, Delta*x, x, dy)
-    float4 b[kBT][kBCh / 2];  // (sigmoid(v), dout*silu'(z)) of channels 2p, 2p+1
 };
 
 template <typename T>
 struct BSmem {
     BRaw<T> raw[kBStages];
-    BConv cv[2];
+    BConv cv;
     float4 hs[kBT][kBThreads];        // recomputed states of the chunk, per lane
     T gx[kBT][kBCh], gdt[kBT][kBCh], gz[kBT][kBCh];   // output tiles (TMA stores)
-    float bc[2][kBT][32];   // per step: slot 8q + j, j < 4 dB[4q+j], else dC[4q+j-4]
+    float bc[kBT][32];   // per step: slot 8q + j, j < 4 dB[4q+j], else dC[4q+j-4]
     uint64_t full[kBStages];
 };
 
@@ -122,30 +125,23 @@ __device__ __forceinline__ void bconvert(BConv &cv, const BRaw<T> &r, int cp, in
     for (int k = 0; k < kBT / 8; ++k) {
         const int t = th + 8 * k;
         const int c = 2 * cp;
-        float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f), a1 = a0, bb = a0;
+        float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f), a1 = a0;
         if (ok && t0 + t < L) {
             const float2 xv = ld_pair(&r.x[t][c]);
             const float2 dv = ld_pair(&r.dt[t][c]);
             const float2 ov = ld_pair(&r.dout[t][c]);
-            const float v0 = dv.x + bias.x, v1 = dv.y + bias.y;
-            const float d0 = softplus(v0), d1 = softplus(v1);   // as in the forward
-            float dy0 = ov.x, dy1 = ov.y, q0 = 0.f, q1 = 0.f;
+            const float d0 = softplus(dv.x + bias.x), d1 = softplus(dv.y + bias.y);   // as in the forward
+            float dy0 = ov.x, dy1 = ov.y;
             if (gate) {
                 const float2 zv = ld_pair(&r.z[t][c]);
-                const float s0 = __fdividef(1.f, 1.f + ex2(-zv.x * kLog2e));
-                const float s1 = __fdividef(1.f, 1.f + ex2(-zv.y * kLog2e));
-                dy0 = ov.x * zv.x * s0;
-                dy1 = ov.y * zv.y * s1;
-                q0 = ov.x * s0 * fmaf(zv.x, 1.f - s0, 1.f);
-                q1 = ov.y * s1 * fmaf(zv.y, 1.f - s1, 1.f);
+                dy0 = ov.x * silu(zv.x);
+                dy1 = ov.y * silu(zv.y);
             }
             a0 = make_float4(d0, d0 * xv.x, xv.x, dy0);
             a1 = make_float4(d1, d1 * xv.y, xv.y, dy1);
-            bb = make_float4(sigmoid_v(v0), q0, sigmoid_v(v1), q1);
         }
         cv.a[t][c] = a0;
         cv.a[t][c + 1] = a1;
-        cv.b[t][cp] = bb;
     }
 }
 
@@ -191,6 +187,7 @@ __device__ __forceinline__ void store_out(T (&tile)[kBT][kBCh], int t, int c, fl
 // buffer for its next use (thread: step tid / 8, slots 4 sg .. 4 sg + 3).
 __device__ __forceinline__ void flush_bc(float (&bc)[kBT][32], const GradParams &g, int64_t b, int64_t t0,
                                          int64_t L) {
+    static_assert(kBT * 8 == kBThreads, "one thread per step and slot group");
     const int t = threadIdx.x >> 3, sg = threadIdx.x & 7;
     float4 &v = *reinterpret_cast<float4 *>(&bc[t][4 * sg]);
     if (t0 + t < L) {
@@ -202,7 +199,7 @@ __device__ __forceinline__ void flush_bc(float (&bc)[kBT][32], const GradParams 
 }
 
 template <typename T>
-__global__ void __launch_bounds__(kBThreads, 3) backward_kernel(const __grid_constant__ BwdArgs a) {
+__global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_constant__ BwdArgs a) {
     constexpr int S = kBStages;
     extern __shared__ unsigned char smem_dyn[];
     BSmem<T> &s = *reinterpret_cast<BSmem<T> *>((reinterpret_cast<uintptr_t>(smem_dyn) + 127) &
@@ -221,7 +218,7 @@ __global__ void __launch_bounds__(kBThreads, 3) backward_kernel(const __grid_con
         for (int st = 0; st < S; ++st) mbar_init(&s.full[st], 1);
         fence_mbar_init();
     }
-    for (int i = tid; i < 2 * kBT * 32; i += kBThreads) (&s.bc[0][0][0])[i] = 0.f;
+    for (int i = tid; i < kBT * 32; i += kBThreads) (&s.bc[0][0])[i] = 0.f;
     __syncthreads();
     // ring slot j holds chunk nchunks-1-j (reverse order)
     if (tid == 0)
@@ -240,7 +237,7 @@ __global__ void __launch_bounds__(kBThreads, 3) backward_kernel(const __grid_con
     const int64_t d = d0 + c;
     const bool chan_ok = d < D;
     float2 a2[2], Ar[2], g[2], dA[2];
-    float dsk = 0.f, dD_acc = 0.f, db_acc = 0.f;
+    float dsk = 0.f, dtb = 0.f, dD_acc = 0.f, db_acc = 0.f;
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
         a2[k] = make_float2(0.f, 0.f); Ar[k] = a2[k]; g[k] = a2[k]; dA[k] = a2[k];
@@ -252,6 +249,7 @@ __global__ void __launch_bounds__(kBThreads, 3) backward_kernel(const __grid_con
         a2[0] = make_float2(av.x * kLog2e, av.y * kLog2e);
         a2[1] = make_float2(av.z * kLog2e, av.w * kLog2e);
         dsk = p.D ? __ldg(p.D + d) : 0.f;
+        dtb = p.dt_bias ? __ldg(p.dt_bias + d) : 0.f;
         if (gp.dh_last) {
             const float4 gv = __ldg(reinterpret_cast<const float4 *>(gp.dh_last + ((int64_t)b * D + d) * kDState + 4 * q));
             g[0] = make_float2(gv.x, gv.y);
@@ -259,39 +257,40 @@ __global__ void __launch_bounds__(kBThreads, 3) backward_kernel(const __grid_con
         }
     }
 
-    // ---- prologue: convert the last chunk
-    bool ok = mbar_wait(&s.full[0], 0);
-    if (ok) bconvert(s.cv[0], s.raw[0], cp, th, bias2, cok, (nchunks - 1) * kBT, L, gate);
-    if (__syncthreads_or(ok ? 0 : 1)) {
-        if (tid == 0) {
-            report(p.status, 4 /* MB_ERR_TIMEOUT */, 0);
-            for (int j = 0; j < S && j < nchunks; ++j) mbar_wait(&s.full[j], 0);
-        }
-        return;
-    }
+    // checkpoint of chunk i, loaded one iteration ahead (its latency overlaps
+    // the previous chunk's sweep)
+    auto load_ckpt = [&](int64_t i) {
+        return chan_ok ? __ldg(reinterpret_cast<const float4 *>(
+                             gp.h_ckpt + (((int64_t)b * nchunks + i) * D + d) * kDState + 4 * q))
+                       : make_float4(0.f, 0.f, 0.f, 0.f);
+    };
+    float4 ck_next = load_ckpt(nchunks - 1);
 
+    bool ok = true;
     for (int64_t j = 0; j < nchunks; ++j) {
         const int64_t i = nchunks - 1 - j;   // chunk of this iteration
         const int64_t t0 = i * kBT;
-        // (1) the next chunk (i - 1): wait for its tiles, convert
-        if (j + 1 < nchunks) {
-            const int64_t jn = j + 1;
-            ok = mbar_wait(&s.full[jn % S], (uint32_t)((jn / S) & 1));
-            if (ok) bconvert(s.cv[jn & 1], s.raw[jn % S], cp, th, bias2, cok, t0 - kBT, L, gate);
+        // (1) wait for chunk i's tiles and convert them; dB, dC of chunk i + 1
+        ok = mbar_wait(&s.full[j % S], (uint32_t)((j / S) & 1));
+        if (ok) bconvert(s.cv, s.raw[j % S], cp, th, bias2, cok, t0, L, gate);
+        if (j >= 1) flush_bc(s.bc, gp, b, t0 + kBT, L);
+        if (__syncthreads_or(ok ? 0 : 1)) {
+            if (tid == 0) {
+                report(p.status, 4 /* MB_ERR_TIMEOUT */, j);
+                int64_t last = j + S - 1;   // ring slots issued so far: 0 .. j+S-1
+                if (last > nchunks - 1) last = nchunks - 1;
+                for (int64_t jj = j; jj <= last; ++jj)
+                    mbar_wait(&s.full[jj % S], (uint32_t)((jj / S) & 1));
+                bulk_wait_all();
+            }
+            return;
         }
-        // (1b) dB, dC of the previous iteration's chunk (i + 1)
-        if (j >= 1) flush_bc(s.bc[(j - 1) & 1], gp, b, t0 + kBT, L);
 
         // (2) chunk i
-        const BConv &cv = s.cv[j & 1];
+        const BConv &cv = s.cv;
         const BRaw<T> &rs = s.raw[j % S];
-        float2 hc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-        if (chan_ok) {
-            const float4 hv = __ldg(reinterpret_cast<const float4 *>(
-                gp.h_ckpt + (((int64_t)b * nchunks + i) * D + d) * kDState + 4 * q));
-            hc[0] = make_float2(hv.x, hv.y);
-            hc[1] = make_float2(hv.z, hv.w);
-        }
+        const float2 hc[2] = {make_float2(ck_next.x, ck_next.y), make_float2(ck_next.z, ck_next.w)};
+        if (i > 0) ck_next = load_ckpt(i - 1);
         // recompute the chunk's forward states (same arithmetic as the forward)
         float4(&hs)[kBT][kBThreads] = s.hs;
         float yv[kBT / 4];   // lane q: share-summed y of step 4m + q
@@ -314,7 +313,7 @@ __global__ void __launch_bounds__(kBThreads, 3) backward_kernel(const __grid_con
             }
         }
         // reverse sweep over the chunk
-        float (&bcs)[kBT][32] = s.bc[j & 1];
+        float (&bcs)[kBT][32] = s.bc;
         float s1[4], s2[4];
         float4 hcur = hs[kBT - 1][tid];   // h_t; h_{t-1} is loaded each step
 #pragma unroll
@@ -351,8 +350,14 @@ __global__ void __launch_bounds__(kBThreads, 3) backward_kernel(const __grid_con
                 const float S2 = reduce4(s2[0], s2[1], s2[2], s2[3], q);
                 const int tq = t + q;
                 const float4 aq = cv.a[tq][c];
-                const float4 bq = cv.b[tq][c >> 1];
-                const float sig = (c & 1) ? bq.z : bq.x, qz = (c & 1) ? bq.w : bq.y;
+                const bool live = chan_ok && t0 + tq < L;
+                const float sig = live ? sigmoid_v(to_f32(rs.dt[tq][c]) + dtb) : 0.f;
+                float qz = 0.f;
+                if (gate && live) {
+                    const float zt = to_f32(rs.z[tq][c]);
+                    const float sz = __fdividef(1.f, 1.f + ex2(-zt * kLog2e));
+                    qz = to_f32(rs.dout[tq][c]) * sz * fmaf(zt, 1.f - sz, 1.f);
+                }
                 const float dx = fmaf(aq.x, S1, aq.w * dsk);
                 const float ddt = fmaf(aq.z, S1, S2) * sig;
                 const float y = fmaf(dsk, aq.z, yv[t >> 2]);
@@ -364,17 +369,7 @@ __global__ void __launch_bounds__(kBThreads, 3) backward_kernel(const __grid_con
             }
         }
         fence_proxy_async_smem();   // output tiles -> visible to the TMA stores
-        if (__syncthreads_or(ok ? 0 : 1)) {
-            if (tid == 0) {
-                report(p.status, 4 /* MB_ERR_TIMEOUT */, j + 1);
-                int64_t last = j + S - 1;   // ring slots issued so far: 0 .. max(S-1, j+S-1)
-                if (last > nchunks - 1) last = nchunks - 1;
-                for (int64_t jj = j + 1; jj <= last; ++jj)
-                    mbar_wait(&s.full[jj % S], (uint32_t)((jj / S) & 1));
-                bulk_wait_all();
-            }
-            return;
-        }
+        __syncthreads();
         if (tid == 0) {
             tma_store_3d(&a.tm_dx, &s.gx[0][0], d0, (int)t0, b);
             tma_store_3d(&a.tm_ddt, &s.gdt[0][0], d0, (int)t0, b);
@@ -386,14 +381,13 @@ __global__ void __launch_bounds__(kBThreads, 3) backward_kernel(const __grid_con
                 fence_proxy_async_smem();
                 issue_bchunk(s, a, (int)(j % S), nchunks - 1 - (j + S), d0, b);
             }
-            // the output tiles are rewritten next iteration: wait until these
-            // stores have read them
+            // the output tiles are rewritten after the next conversion
+            // barrier: wait until these stores have read them
             bulk_wait_read_all();
         }
-        __syncthreads();
     }
     // dB, dC of chunk 0
-    flush_bc(s.bc[(nchunks - 1) & 1], gp, b, 0, L);
+    flush_bc(s.bc, gp, b, 0, L);
 
     // per-channel sums: dD, dbias over the 4 lanes of the channel
     dD_acc += __shfl_xor_sync(kFull, dD_acc, 8);
