@@ -19,6 +19,12 @@ def test_algorithmic_bytes_of_the_workloads():
     assert sum(bench.bytes_verify(32, 16, 2048)) == 79_872_000
     assert sum(bench.bytes_rollback(32, 2048)) == 8_388_736
     assert sum(bench.bytes_step(256, 4608)) == 160_780_288
+    # backward: reads 4 token tensors, B, C, parameters, 512 checkpoints, dh_last;
+    # writes 3 token tensors, dB, dC (fp32), dA, dD, ddt_bias, dh0
+    rd, wr = bench.bytes_backward(8, 8192, 2048)
+    st = 8 * 2048 * 16 * 4
+    assert rd == 4 * 8 * 8192 * 2048 * 2 + 2 * 8 * 8192 * 16 * 2 + 2048 * 16 * 4 + 2 * 2048 * 4 + 512 * st + st
+    assert wr == 3 * 8 * 8192 * 2048 * 2 + 2 * 8 * 8192 * 16 * 4 + 2048 * 16 * 4 + 2 * 2048 * 4 + st
     parts = bench.step_bytes()
     assert parts["step"] == 48 * 160_780_288
 
