@@ -227,6 +227,40 @@ mb_status mb_scan_backward(const mb_scan_args *args, const float *h_ckpt, const 
                            const float *dh_last, const mb_scan_grads *grads, void *ws,
                            size_t ws_bytes, void *stream);
 
+/* ------------------------------------------------------------------------
+ * Element-wise steps of the Mamba block around the scan, for recurrent
+ * decoding of a whole MambaByte model (Figure 6; Table 6 "Pre-SSM 1D
+ * convolution"). Rows are [batch, width], contiguous, 16-byte aligned;
+ * width % 8 == 0.
+ * ------------------------------------------------------------------------ */
+
+/*
+ * Residual add and RMS normalisation that open a block:
+ *   residual[b] += add[b]            (skipped when add == NULL)
+ *   out[b] = residual[b] * w / sqrt(mean_j residual[b, j]^2 + eps)
+ * residual: fp32 [batch, width], read and written; add, out: dtype
+ * [batch, width]; w: fp32 [width]. width <= 8192. out must not overlap the
+ * other arguments.
+ */
+mb_status mb_rmsnorm(const void *add, float *residual, const float *w, float eps, void *out,
+                     int64_t batch, int64_t width, int32_t dtype, void *stream);
+
+/*
+ * One decode step of the causal depthwise convolution (kernel size 4) and its
+ * SiLU, the step that feeds the scan's x:
+ *   out[b, d] = silu(w[d,0] s[b,0,d] + w[d,1] s[b,1,d] + w[d,2] s[b,2,d]
+ *                    + w[d,3] x[b,d] + bias[d])
+ * then s[b,0] <- s[b,1], s[b,1] <- s[b,2], s[b,2] <- x[b].
+ *   x, out : [batch, width], dtype
+ *   state  : [batch, 3, width], dtype, the three previous inputs (oldest
+ *            first; zeros at the start of a sequence), read and written
+ *   w      : [width, 4] fp32 (w[d, 3] multiplies the current input);
+ *   bias   : [width] fp32 or NULL
+ * out must not overlap x, state, w or bias.
+ */
+mb_status mb_conv1d_step(const void *x, void *state, const float *w, const float *bias, void *out,
+                         int64_t batch, int64_t width, int32_t dtype, void *stream);
+
 /*
  * Read and clear the status block of a workspace (blocking: waits for
  * `stream`). Returns MB_OK, or the first device-side error recorded by

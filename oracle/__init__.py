@@ -16,6 +16,11 @@ Functions (MambaByte, Eq. 2-3, discretisation appendix, Table 6, Algorithm 1):
                  rank in the verifier's distribution is within top-beta.
 * ``scan_backward`` - every input gradient of J given dJ/dout and dJ/dh_last
                  (the training path), by the adjoint recurrence in fp64.
+* ``rmsnorm``, ``conv1d_step``, ``block_step`` - the Mamba block around the
+                 scan for recurrent decoding (Figure 6, Table 6): residual add
+                 with RMS normalisation, one step of the causal depthwise
+                 convolution with SiLU, and a whole block step (projections as
+                 fp64 matrix products).
 
 Inputs are widened exactly to float64 before the call (bf16 and fp32 values
 are exactly representable in fp64).
@@ -192,3 +197,66 @@ def accept_topk(logits, drafted, beta):
                 break
         out[s] = a
     return out
+
+
+def bf16_round(a):
+    """Round float64 values to the nearest bfloat16 (ties to even), returned
+    as float64: the value a bf16 tensor holds after a cast."""
+    a = np.asarray(a, dtype=np.float64)
+    f = a.astype(np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    lsb = (u >> 16) & 1
+    u = (u + 0x7FFF + lsb) & 0xFFFF0000
+    out = u.astype(np.uint32).view(np.float32).astype(np.float64)
+    return np.where(np.isfinite(f), out, f.astype(np.float64))
+
+
+def rmsnorm(residual, w, eps, add=None):
+    """Residual add and RMS normalisation that open a Mamba block:
+    r = residual + add; out = r / sqrt(mean(r^2) + eps) * w (last axis).
+    Returns (r, out)."""
+    r = _f64(residual) + (0.0 if add is None else _f64(add))
+    out = r / np.sqrt(np.mean(r * r, axis=-1, keepdims=True) + eps) * _f64(w)
+    return r, out
+
+
+def silu(v):
+    v = np.asarray(v, dtype=np.float64)
+    return v / (1.0 + np.exp(-v))
+
+
+def conv1d_step(state, x, w, bias=None):
+    """One decode step of the causal depthwise convolution (kernel 4) with
+    SiLU. state [b, 3, d] holds the three previous inputs, oldest first;
+    x [b, d]; w [d, 4] (w[:, 3] multiplies the current input); bias [d].
+    Returns (out [b, d], new_state)."""
+    state, x, w = _f64(state), _f64(x), _f64(w)
+    acc = state[:, 0] * w[:, 0] + state[:, 1] * w[:, 1] + state[:, 2] * w[:, 2] + x * w[:, 3]
+    if bias is not None:
+        acc = acc + _f64(bias)
+    return silu(acc), np.stack([state[:, 1], state[:, 2], x], axis=1)
+
+
+def block_step(layer, residual, add, ssm_state, conv_state, eps=1e-5, cast=bf16_round):
+    """One Mamba block for one decoded byte per stream (MambaByte's Mamba-1
+    block, Figure 6; Table 6 rows). `layer` holds float64 weights: norm_w,
+    W_in_x, W_in_z [d_inner, d_model], conv_w [d_inner, 4], conv_b, W_dtlow
+    [r, d_inner], W_B, W_C [16, d_inner], W_dt [d_inner, r], dt_bias, A
+    [d_inner, 16], D, W_out [d_model, d_inner]. residual [b, d_model] (fp32
+    stream), add = the previous block's output or None. Tensors the GPU path
+    keeps in the input dtype are passed through `cast` at the same points.
+    Returns (residual, out, ssm_state, conv_state)."""
+    r, h = rmsnorm(residual, layer["norm_w"], eps, add)
+    h = cast(h)
+    x = cast(h @ layer["W_in_x"].T)
+    z = cast(h @ layer["W_in_z"].T)
+    xc, conv_state = conv1d_step(conv_state, x, layer["conv_w"], layer["conv_b"])
+    xc = cast(xc)
+    dtl = cast(xc @ layer["W_dtlow"].T)
+    Bm = cast(xc @ layer["W_B"].T)
+    Cm = cast(xc @ layer["W_C"].T)
+    dt = cast(dtl @ layer["W_dt"].T)
+    y, ssm_state = step(ssm_state, x=xc, dt=dt, B=Bm, C=Cm, A=layer["A"], z=z, D=layer["D"],
+                        dt_bias=layer["dt_bias"])
+    out = cast(cast(y) @ layer["W_out"].T)
+    return r, out, ssm_state, conv_state

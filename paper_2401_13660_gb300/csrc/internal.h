@@ -53,6 +53,11 @@ struct GradParams {
     float *dh0;                   // [batch, d_inner, 16] or null
 };
 cudaError_t launch_backward(const ScanParams &p, const GradParams &g, bool bf16, cudaStream_t s);
+// Block steps around the scan (block.cu).
+cudaError_t launch_rmsnorm(const void *add, float *residual, const float *w, float eps, void *out,
+                           int64_t batch, int64_t width, bool bf16, cudaStream_t s);
+cudaError_t launch_conv_step(const void *x, void *state, const float *w, const float *bias, void *out,
+                             int64_t batch, int64_t width, bool bf16, cudaStream_t s);
 cudaError_t launch_step(const ScanParams &p, bool bf16, cudaStream_t s);
 // One step from the state kept after accept[s] drafted bytes: p.h0 (may be
 // null = zeros) when accept[s] == 0, else h_all[s, accept[s]-1]; the new state

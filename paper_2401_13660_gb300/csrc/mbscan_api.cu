@@ -320,6 +320,46 @@ mb_status mb_scan_backward(const mb_scan_args *args, const float *h_ckpt, const 
     return from_cuda(mbscan::launch_backward(p, gp, args->dtype == MB_BF16, (cudaStream_t)stream));
 }
 
+mb_status mb_rmsnorm(const void *add, float *residual, const float *w, float eps, void *out,
+                     int64_t batch, int64_t width, int32_t dtype, void *stream) {
+    if (batch < 0 || width < 0 || batch > kMaxTokens || width > 8192 || width % 8 != 0)
+        return width > 8192 || width % 8 != 0 ? MB_ERR_UNSUPPORTED : MB_ERR_INVALID_ARG;
+    if (dtype != MB_F32 && dtype != MB_BF16) return MB_ERR_INVALID_ARG;
+    if (batch * width == 0) return MB_OK;
+    if (!(eps >= 0.f)) return MB_ERR_INVALID_ARG;
+    if (!residual || !w || !out || !aligned16(residual) || !aligned16(w) || !aligned16(out) ||
+        (add && !aligned16(add)))
+        return MB_ERR_INVALID_ARG;
+    const int64_t es = dtype == MB_BF16 ? 2 : 4;
+    const Range ro = range_of(out, batch * width * es);
+    if (overlap(ro, range_of(residual, batch * width * 4)) || overlap(ro, range_of(w, width * 4)) ||
+        overlap(ro, range_of(add, batch * width * es)) ||
+        overlap(range_of(residual, batch * width * 4), range_of(add, batch * width * es)))
+        return MB_ERR_INVALID_ARG;
+    return from_cuda(mbscan::launch_rmsnorm(add, residual, w, eps, out, batch, width, dtype == MB_BF16,
+                                            (cudaStream_t)stream));
+}
+
+mb_status mb_conv1d_step(const void *x, void *state, const float *w, const float *bias, void *out,
+                         int64_t batch, int64_t width, int32_t dtype, void *stream) {
+    if (batch < 0 || width < 0 || batch > kMaxTokens || width > kMaxTokens) return MB_ERR_INVALID_ARG;
+    if (width % 8 != 0) return MB_ERR_UNSUPPORTED;
+    if (dtype != MB_F32 && dtype != MB_BF16) return MB_ERR_INVALID_ARG;
+    if (batch * width == 0) return MB_OK;
+    if (batch > kMaxTokens / width) return MB_ERR_INVALID_ARG;
+    if (!x || !state || !w || !out || !aligned16(x) || !aligned16(state) || !aligned16(w) ||
+        !aligned16(out) || (bias && !aligned16(bias)))
+        return MB_ERR_INVALID_ARG;
+    const int64_t es = dtype == MB_BF16 ? 2 : 4;
+    const Range ro = range_of(out, batch * width * es), rs = range_of(state, batch * 3 * width * es);
+    const Range rx = range_of(x, batch * width * es);
+    if (overlap(ro, rx) || overlap(ro, rs) || overlap(rs, rx) || overlap(ro, range_of(w, width * 16)) ||
+        overlap(ro, range_of(bias, width * 4)))
+        return MB_ERR_INVALID_ARG;
+    return from_cuda(mbscan::launch_conv_step(x, state, w, bias, out, batch, width, dtype == MB_BF16,
+                                              (cudaStream_t)stream));
+}
+
 mb_status mb_check(void *ws, void *stream, int64_t *detail) {
     if (detail) *detail = -1;
     if (ws == nullptr) return MB_ERR_INVALID_ARG;

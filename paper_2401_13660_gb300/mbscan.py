@@ -77,9 +77,12 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
             lib.mb_accept_topk.argtypes = [vp, ctypes.c_int32, vp, i64, i64, ctypes.c_int32, vp, vp]
             lib.mb_step_resume.argtypes = [ap, vp, vp, i64, vp, vp, sz, vp]
             lib.mb_scan_prefill_ckpt.argtypes = [ap, vp, vp, vp, sz, vp]
+            lib.mb_rmsnorm.argtypes = [vp, vp, vp, ctypes.c_float, vp, i64, i64, ctypes.c_int32, vp]
+            lib.mb_conv1d_step.argtypes = [vp, vp, vp, vp, vp, i64, i64, ctypes.c_int32, vp]
             lib.mb_scan_backward.argtypes = [ap, vp, vp, vp, ctypes.POINTER(mb_scan_grads), vp, sz, vp]
             for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_check",
-                      "mb_accept_topk", "mb_step_resume", "mb_scan_prefill_ckpt", "mb_scan_backward"):
+                      "mb_accept_topk", "mb_step_resume", "mb_scan_prefill_ckpt", "mb_scan_backward",
+                      "mb_rmsnorm", "mb_conv1d_step"):
                 getattr(lib, f).restype = ctypes.c_int
             lib.mb_status_string.argtypes = [ctypes.c_int]
             lib.mb_status_string.restype = ctypes.c_char_p
@@ -269,6 +272,42 @@ def mb_scan_backward(x, dt, B, C, A, h_ckpt, dout, *, z=None, D=None, dt_bias=No
                                          ctypes.byref(st), _ptr(ws), ws.numel(), _stream(stream))
     _check(rc, "mb_scan_backward")
     return g
+
+
+def mb_rmsnorm(residual, w, out, *, add=None, eps=1e-5, stream=None):
+    """residual [batch, width] fp32 += add (if given); out = residual * w /
+    rms(residual), out and add in the input dtype (fp32 or bf16)."""
+    if out.dtype not in _DTYPES:
+        raise TypeError(f"unsupported dtype {out.dtype}")
+    batch, width = residual.shape
+    dev = residual.device
+    _need(residual, "residual", torch.float32, (batch, width), dev)
+    _need(w, "w", torch.float32, (width,), dev)
+    _need(out, "out", out.dtype, (batch, width), dev)
+    _need(add, "add", out.dtype, (batch, width), dev)
+    rc = load_library().mb_rmsnorm(_ptr(add), _ptr(residual), _ptr(w), float(eps), _ptr(out), batch, width,
+                                   _DTYPES[out.dtype], _stream(stream))
+    _check(rc, "mb_rmsnorm")
+    return out
+
+
+def mb_conv1d_step(x, state, w, out, *, bias=None, stream=None):
+    """One causal depthwise convolution step (kernel 4) with SiLU: x, out
+    [batch, width]; state [batch, 3, width] (previous inputs, oldest first),
+    updated in place; w [width, 4] fp32; bias [width] fp32."""
+    if x.dtype not in _DTYPES:
+        raise TypeError(f"unsupported dtype {x.dtype}")
+    batch, width = x.shape
+    dev = x.device
+    _need(x, "x", x.dtype, (batch, width), dev)
+    _need(state, "state", x.dtype, (batch, 3, width), dev)
+    _need(w, "w", torch.float32, (width, 4), dev)
+    _need(bias, "bias", torch.float32, (width,), dev)
+    _need(out, "out", x.dtype, (batch, width), dev)
+    rc = load_library().mb_conv1d_step(_ptr(x), _ptr(state), _ptr(w), _ptr(bias), _ptr(out), batch, width,
+                                       _DTYPES[x.dtype], _stream(stream))
+    _check(rc, "mb_conv1d_step")
+    return out
 
 
 def mb_step_resume(x, dt, B, C, A, y, h_all, accept, state, *, z=None, D=None, dt_bias=None, h0=None,

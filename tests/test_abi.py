@@ -194,6 +194,24 @@ def test_training_path_checks():
     assert bwd(args=nz, g=grads(dz=None, dD=None, ddt_bias=None, dh0=None)) in want_launch
 
 
+def test_block_kernel_checks():
+    lib = mb.load_library()
+    res, w, out, add = FAKE, FAKE + (1 << 32), FAKE + (2 << 32), FAKE + (3 << 32)
+    f = ctypes.c_float(1e-5)
+    assert lib.mb_rmsnorm(add, res, w, f, out, 4, 64, mb.MB_BF16, None) in (mb.MB_OK, mb.MB_ERR_CUDA)
+    assert lib.mb_rmsnorm(add, res, w, f, out, 4, 60, mb.MB_BF16, None) == mb.MB_ERR_UNSUPPORTED
+    assert lib.mb_rmsnorm(add, res, w, f, out, 4, 8200, mb.MB_BF16, None) == mb.MB_ERR_UNSUPPORTED
+    assert lib.mb_rmsnorm(add, res, w, f, res + 64, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_rmsnorm(add, res, w, ctypes.c_float(-1.0), out, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_rmsnorm(add, None, w, f, out, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
+    x, st, cw, cb, co = FAKE, FAKE + (1 << 32), FAKE + (2 << 32), FAKE + (3 << 32), FAKE + (4 << 32)
+    assert lib.mb_conv1d_step(x, st, cw, cb, co, 4, 12, mb.MB_BF16, None) == mb.MB_ERR_UNSUPPORTED
+    assert lib.mb_conv1d_step(x, st, cw, cb, st + 16, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_conv1d_step(x, x + 32, cw, cb, co, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_conv1d_step(x, st, None, cb, co, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_conv1d_step(x, st, cw, cb, co, 0, 64, mb.MB_BF16, None) == mb.MB_OK
+
+
 def test_binding_rejects_cpu_shape_errors():
     import torch
     x = torch.zeros(1, 4, 8, dtype=torch.bfloat16)
