@@ -58,7 +58,13 @@ typedef enum { MB_F32 = 0, MB_BF16 = 1 } mb_dtype;
  *   x, z, dt : [batch, seqlen, d_inner], dtype. dt is the pre-softplus
  *              timestep (W_Delta W_R x in Eq. 3). z is the gate input; NULL
  *              means no gate (y = C.h + D x).
- *   B, C     : [batch, seqlen, d_state], dtype (W_B x and W_C x in Eq. 3)
+ *   B, C     : [batch, seqlen, d_state], dtype (W_B x and W_C x in Eq. 3);
+ *              row (b, t) starts bc_stride elements after row (b, t-1)
+ *   bc_stride: elements between consecutive (b, t) rows of B and of C; 0
+ *              means d_state (contiguous). Otherwise >= d_state with
+ *              bc_stride * element size a multiple of 16 bytes: B and C may
+ *              then be column blocks of one wider row, e.g. of the
+ *              [dt_low | B | C] output of a single x-projection GEMM.
  *   A        : [d_inner, d_state] fp32, the diagonal of A per channel
  *   D        : [d_inner] fp32 skip weight; NULL means 0
  *   dt_bias  : [d_inner] fp32 added to dt before softplus; NULL means 0
@@ -68,7 +74,7 @@ typedef enum { MB_F32 = 0, MB_BF16 = 1 } mb_dtype;
 typedef struct {
     int64_t batch, seqlen, d_inner, d_state;
     int32_t dtype;
-    int32_t reserved;
+    int32_t bc_stride;
     const void *x, *z, *dt;
     const void *B, *C;
     const float *A;
@@ -239,7 +245,7 @@ mb_status mb_scan_backward(const mb_scan_args *args, const float *h_ckpt, const 
  *   residual[b] += add[b]            (skipped when add == NULL)
  *   out[b] = residual[b] * w / sqrt(mean_j residual[b, j]^2 + eps)
  * residual: fp32 [batch, width], read and written; add, out: dtype
- * [batch, width]; w: fp32 [width]. width <= 8192. out must not overlap the
+ * [batch, width]; w: fp32 [width]. out must not overlap the
  * other arguments.
  */
 mb_status mb_rmsnorm(const void *add, float *residual, const float *w, float eps, void *out,

@@ -409,10 +409,11 @@ __global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_con
 }
 
 bool make_map3(CUtensorMap *m, const void *base, bool bf16, int64_t batch, int64_t L, int64_t inner,
-               int box_inner) {
+               int box_inner, int64_t row = 0) {
     const int64_t es = bf16 ? 2 : 4;
+    if (row == 0) row = inner;
     const uint64_t dims[3] = {(uint64_t)inner, (uint64_t)L, (uint64_t)batch};
-    const uint64_t strides[2] = {(uint64_t)(inner * es), (uint64_t)(L * inner * es)};
+    const uint64_t strides[2] = {(uint64_t)(row * es), (uint64_t)(L * row * es)};
     const uint32_t box[3] = {(uint32_t)box_inner, (uint32_t)kBT, 1};
     return encode_tmap(m, base, (int)es, 3, dims, strides, box);
 }
@@ -429,8 +430,8 @@ cudaError_t launch_backward_typed(const ScanParams &p, const GradParams &g, cuda
     if (!make_map3(&a.tm_dt, p.dt, bf16, Bn, L, D, kBCh) || !make_map3(&a.tm_x, p.x, bf16, Bn, L, D, kBCh) ||
         (p.z && !make_map3(&a.tm_z, p.z, bf16, Bn, L, D, kBCh)) ||
         !make_map3(&a.tm_dout, g.dout, bf16, Bn, L, D, kBCh) ||
-        !make_map3(&a.tm_B, p.B, bf16, Bn, L, kDState, kDState) ||
-        !make_map3(&a.tm_C, p.C, bf16, Bn, L, kDState, kDState) ||
+        !make_map3(&a.tm_B, p.B, bf16, Bn, L, kDState, kDState, p.bc_stride) ||
+        !make_map3(&a.tm_C, p.C, bf16, Bn, L, kDState, kDState, p.bc_stride) ||
         !make_map3(&a.tm_dx, g.dx, bf16, Bn, L, D, kBCh) || !make_map3(&a.tm_ddt, g.ddt, bf16, Bn, L, D, kBCh) ||
         (p.z && !make_map3(&a.tm_dz, g.dz, bf16, Bn, L, D, kBCh)))
         return cudaErrorInvalidValue;

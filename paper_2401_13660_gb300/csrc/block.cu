@@ -53,35 +53,35 @@ __device__ __forceinline__ void store8(float *p, const float (&v)[8]) {
     reinterpret_cast<float4 *>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
 }
 
-constexpr int kNormThreads = 256;
-
 // residual[b] += add[b] (when given); out[b] = residual[b] / sqrt(mean(residual[b]^2) + eps) * w.
-// One CTA per row; each thread owns 8-element groups g = tid, tid + 256, ...
+// One CTA per row, blockDim = 32 * ceil(groups / 32) (<= 1024) so that each
+// thread usually owns one 8-element group, which it keeps in registers
+// between the sum of squares and the scaling; wider rows loop and re-read.
 template <typename T>
-__global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const T *__restrict__ add, float *residual,
-                                                               const float *__restrict__ w, float eps,
-                                                               T *__restrict__ out, int64_t width) {
-    __shared__ float red[kNormThreads / 32];
+__global__ void __launch_bounds__(1024) rmsnorm_kernel(const T *__restrict__ add, float *residual,
+                                                       const float *__restrict__ w, float eps,
+                                                       T *__restrict__ out, int64_t width) {
+    __shared__ float red[32];
     const int64_t row = blockIdx.x;
     float *r = residual + row * width;
     const int groups = (int)(width / 8);
-    constexpr int kMaxGroups = 4;   // width <= 8 * 256 * 4 = 8192
-    float v[kMaxGroups][8];
+    float v0[8];
     float ss = 0.f;
+    for (int g = threadIdx.x; g < groups; g += blockDim.x) {
+        float v[8];
+        ld8(r + 8 * g, v);
+        if (add) {
+            float a[8];
+            load8(add + row * width + 8 * g, a);
 #pragma unroll
-    for (int k = 0; k < kMaxGroups; ++k) {
-        const int g = threadIdx.x + k * kNormThreads;
-        if (g < groups) {
-            ld8(r + 8 * g, v[k]);
-            if (add) {
-                float a[8];
-                load8(add + row * width + 8 * g, a);
+            for (int j = 0; j < 8; ++j) v[j] += a[j];
+            store8(r + 8 * g, v);
+        }
 #pragma unroll
-                for (int j = 0; j < 8; ++j) v[k][j] += a[j];
-                store8(r + 8 * g, v[k]);
-            }
+        for (int j = 0; j < 8; ++j) ss = fmaf(v[j], v[j], ss);
+        if (g == (int)threadIdx.x) {
 #pragma unroll
-            for (int j = 0; j < 8; ++j) ss = fmaf(v[k][j], v[k][j], ss);
+            for (int j = 0; j < 8; ++j) v0[j] = v[j];
         }
     }
 #pragma unroll
@@ -89,29 +89,31 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const T *__restri
     if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
     __syncthreads();
     float tot = 0.f;
-#pragma unroll
-    for (int i = 0; i < kNormThreads / 32; ++i) tot += red[i];
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) tot += red[i];
     const float scale = rsqrtf(tot / (float)width + eps);
+    for (int g = threadIdx.x; g < groups; g += blockDim.x) {
+        float v[8], wv[8], o[8];
+        if (g == (int)threadIdx.x) {
 #pragma unroll
-    for (int k = 0; k < kMaxGroups; ++k) {
-        const int g = threadIdx.x + k * kNormThreads;
-        if (g < groups) {
-            float wv[8], o[8];
-            load8(w + 8 * g, wv);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) o[j] = v[k][j] * scale * wv[j];
-            store8(out + row * width + 8 * g, o);
+            for (int j = 0; j < 8; ++j) v[j] = v0[j];
+        } else {
+            ld8(r + 8 * g, v);
         }
+        load8(w + 8 * g, wv);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) o[j] = v[j] * scale * wv[j];
+        store8(out + row * width + 8 * g, o);
     }
 }
 
 constexpr int kConvThreads = 256;
+constexpr int kConvRows = 4;   // batch rows per thread (the weights are loaded once for them)
 
 // One decode step of the causal depthwise convolution (kernel 4) and SiLU:
 //   out[b,d] = silu(sum_{j<3} w[d,j] state[b,j,d] + w[d,3] x[b,d] + bias[d]),
 // then the window moves: state[b,0] <- state[b,1], state[b,1] <- state[b,2],
 // state[b,2] <- x[b]. state: [batch, 3, width] in the input dtype (the last
-// three inputs, oldest first). Thread: 8 channels of one row.
+// three inputs, oldest first). Thread: 8 channels of kConvRows rows.
 template <typename T>
 __global__ void __launch_bounds__(kConvThreads) conv_step_kernel(const T *__restrict__ x, T *state,
                                                                  const float *__restrict__ w,
@@ -119,31 +121,39 @@ __global__ void __launch_bounds__(kConvThreads) conv_step_kernel(const T *__rest
                                                                  T *__restrict__ out, int64_t batch,
                                                                  int64_t width) {
     const int64_t groups = width / 8;
+    const int64_t rowblocks = (batch + kConvRows - 1) / kConvRows;
     const int64_t i = (int64_t)blockIdx.x * kConvThreads + threadIdx.x;
-    if (i >= batch * groups) return;
-    const int64_t b = i / groups, d0 = (i - b * groups) * 8;
-    float xv[8], s0[8], s1[8], s2[8], bv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    load8(x + b * width + d0, xv);
-    T *st = state + b * 3 * width + d0;
-    ld8(st, s0);
-    ld8(st + width, s1);
-    ld8(st + 2 * width, s2);
-    if (bias) load8(bias + d0, bv);
-    float o[8];
+    if (i >= rowblocks * groups) return;
+    const int64_t rb = i / groups, d0 = (i - rb * groups) * 8;
+    float4 wj[8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const float4 wj = __ldg(reinterpret_cast<const float4 *>(w + (d0 + j) * 4));
-        float acc = bv[j];
-        acc = fmaf(wj.x, s0[j], acc);
-        acc = fmaf(wj.y, s1[j], acc);
-        acc = fmaf(wj.z, s2[j], acc);
-        acc = fmaf(wj.w, xv[j], acc);
-        o[j] = silu(acc);
+    for (int j = 0; j < 8; ++j) wj[j] = __ldg(reinterpret_cast<const float4 *>(w + (d0 + j) * 4));
+    float bv[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    if (bias) load8(bias + d0, bv);
+#pragma unroll
+    for (int u = 0; u < kConvRows; ++u) {
+        const int64_t b = rb * kConvRows + u;
+        if (b >= batch) break;
+        float xv[8], s0[8], s1[8], s2[8], o[8];
+        load8(x + b * width + d0, xv);
+        T *st = state + b * 3 * width + d0;
+        ld8(st, s0);
+        ld8(st + width, s1);
+        ld8(st + 2 * width, s2);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            float acc = bv[j];
+            acc = fmaf(wj[j].x, s0[j], acc);
+            acc = fmaf(wj[j].y, s1[j], acc);
+            acc = fmaf(wj[j].z, s2[j], acc);
+            acc = fmaf(wj[j].w, xv[j], acc);
+            o[j] = silu(acc);
+        }
+        store8(out + b * width + d0, o);
+        store8(st, s1);
+        store8(st + width, s2);
+        store8(st + 2 * width, xv);
     }
-    store8(out + b * width + d0, o);
-    store8(st, s1);
-    store8(st + width, s2);
-    store8(st + 2 * width, xv);
 }
 
 }  // namespace
@@ -151,18 +161,20 @@ __global__ void __launch_bounds__(kConvThreads) conv_step_kernel(const T *__rest
 cudaError_t launch_rmsnorm(const void *add, float *residual, const float *w, float eps, void *out,
                            int64_t batch, int64_t width, bool bf16, cudaStream_t s) {
     if (batch == 0 || width == 0) return cudaSuccess;
+    const int64_t groups = width / 8;
+    const unsigned threads = (unsigned)(groups >= 1024 ? 1024 : 32 * ((groups + 31) / 32));
     if (bf16)
-        rmsnorm_kernel<__nv_bfloat16><<<(unsigned)batch, kNormThreads, 0, s>>>(
+        rmsnorm_kernel<__nv_bfloat16><<<(unsigned)batch, threads, 0, s>>>(
             static_cast<const __nv_bfloat16 *>(add), residual, w, eps, static_cast<__nv_bfloat16 *>(out), width);
     else
-        rmsnorm_kernel<float><<<(unsigned)batch, kNormThreads, 0, s>>>(
-            static_cast<const float *>(add), residual, w, eps, static_cast<float *>(out), width);
+        rmsnorm_kernel<float><<<(unsigned)batch, threads, 0, s>>>(static_cast<const float *>(add), residual, w, eps,
+                                                                  static_cast<float *>(out), width);
     return cudaGetLastError();
 }
 
 cudaError_t launch_conv_step(const void *x, void *state, const float *w, const float *bias, void *out,
                              int64_t batch, int64_t width, bool bf16, cudaStream_t s) {
-    const int64_t n = batch * (width / 8);
+    const int64_t n = ((batch + kConvRows - 1) / kConvRows) * (width / 8);
     if (n == 0) return cudaSuccess;
     const unsigned grid = (unsigned)((n + kConvThreads - 1) / kConvThreads);
     if (bf16)

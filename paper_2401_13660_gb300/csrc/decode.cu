@@ -281,7 +281,7 @@ cudaError_t launch_step_typed(const ScanParams &p, const float *h_all, const int
     const uint64_t tstr[1] = {(uint64_t)p.d_inner * es};
     const uint32_t tbox[2] = {kStepCh, kStepRows};
     const uint64_t bdims[2] = {kDState, (uint64_t)p.batch};
-    const uint64_t bstr[1] = {(uint64_t)kDState * es};
+    const uint64_t bstr[1] = {(uint64_t)p.bc_stride * es};
     const uint32_t bbox[2] = {kDState, kStepRows};
     bool ok_maps = true;
     if constexpr (kResume) {

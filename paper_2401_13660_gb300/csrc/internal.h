@@ -20,6 +20,7 @@ constexpr size_t kStatusBytes = 256;
 struct ScanParams {
     int64_t batch, seqlen, d_inner;  // d_state is fixed to 16
     const void *x, *z, *dt, *B, *C;
+    int64_t bc_stride;   // elements between consecutive (b, t) rows of B and C (>= 16)
     const float *A, *D, *dt_bias, *h0;
     void *y;
     float *h_out;      // prefill: h_last (may be null); verify: h_all; step: state

@@ -30,6 +30,15 @@ bool overlap(Range a, Range b) { return a.lo < b.hi && b.lo < a.hi && a.lo != a.
 // 32-bit element counts the kernels assume for token tensors.
 constexpr int64_t kMaxTokens = (int64_t)1 << 31;
 
+// Bytes spanned by B (or C): rows bc_stride elements apart.
+int64_t bc_bytes(const mb_scan_args *a) {
+    const int64_t rows = a->batch * a->seqlen;
+    if (rows <= 0) return 0;
+    const int64_t es = a->dtype == MB_BF16 ? 2 : 4;
+    const int64_t stride = a->bc_stride ? a->bc_stride : a->d_state;
+    return ((rows - 1) * stride + a->d_state) * es;
+}
+
 // Validate the common part of a scan problem; `need_seqlen1` for mb_step.
 mb_status check_args(const mb_scan_args *a, bool need_seqlen1, bool need_y = true) {
     if (a == nullptr) return MB_ERR_INVALID_ARG;
@@ -37,6 +46,9 @@ mb_status check_args(const mb_scan_args *a, bool need_seqlen1, bool need_y = tru
     if (a->dtype != MB_F32 && a->dtype != MB_BF16) return MB_ERR_INVALID_ARG;
     if (need_seqlen1 && a->seqlen != 1) return MB_ERR_INVALID_ARG;
     if (a->d_state != mbscan::kDState) return MB_ERR_UNSUPPORTED;
+    if (a->bc_stride != 0 && (a->bc_stride < a->d_state ||
+                              (a->bc_stride * (a->dtype == MB_BF16 ? 2 : 4)) % 16 != 0))
+        return MB_ERR_INVALID_ARG;
     if (a->d_inner % 8 != 0) return MB_ERR_UNSUPPORTED;
     if (a->batch > kMaxTokens || a->seqlen > kMaxTokens || a->d_inner > kMaxTokens)
         return MB_ERR_INVALID_ARG;
@@ -53,7 +65,7 @@ mb_status check_args(const mb_scan_args *a, bool need_seqlen1, bool need_y = tru
     // y must not overlap any input.
     const int64_t es = a->dtype == MB_BF16 ? 2 : 4;
     const int64_t tok = a->batch * a->seqlen * a->d_inner * es;
-    const int64_t bc = a->batch * a->seqlen * a->d_state * es;
+    const int64_t bc = bc_bytes(a);
     const Range ry = range_of(a->y, tok);
     const Range ins[] = {range_of(a->x, tok), range_of(a->z, tok), range_of(a->dt, tok),
                          range_of(a->B, bc), range_of(a->C, bc),
@@ -71,6 +83,7 @@ ScanParams to_params(const mb_scan_args *a, float *h_out, StatusBlock *status) {
     p.seqlen = a->seqlen;
     p.d_inner = a->d_inner;
     p.x = a->x; p.z = a->z; p.dt = a->dt; p.B = a->B; p.C = a->C;
+    p.bc_stride = a->bc_stride ? a->bc_stride : a->d_state;
     p.A = a->A; p.D = a->D; p.dt_bias = a->dt_bias; p.h0 = a->h0;
     p.y = a->y;
     p.h_out = h_out;
@@ -190,8 +203,8 @@ mb_status mb_step(const mb_scan_args *args, float *state, void *stream) {
     const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
     const int64_t tok = chans * es;
     const Range others[] = {range_of(args->y, tok), range_of(args->x, tok), range_of(args->z, tok),
-                            range_of(args->dt, tok), range_of(args->B, args->batch * args->d_state * es),
-                            range_of(args->C, args->batch * args->d_state * es),
+                            range_of(args->dt, tok), range_of(args->B, bc_bytes(args)),
+                            range_of(args->C, bc_bytes(args)),
                             range_of(args->A, args->d_inner * args->d_state * 4)};
     for (const Range &r : others)
         if (overlap(rs, r)) return MB_ERR_INVALID_ARG;
@@ -218,8 +231,8 @@ mb_status mb_step_resume(const mb_scan_args *args, const float *h_all, const int
     const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
     const int64_t tok = chans * es;
     const Range others[] = {range_of(args->y, tok), range_of(args->x, tok), range_of(args->z, tok),
-                            range_of(args->dt, tok), range_of(args->B, args->batch * args->d_state * es),
-                            range_of(args->C, args->batch * args->d_state * es),
+                            range_of(args->dt, tok), range_of(args->B, bc_bytes(args)),
+                            range_of(args->C, bc_bytes(args)),
                             range_of(args->A, args->d_inner * args->d_state * 4),
                             range_of(h_all, args->batch * k * per), range_of(accept, args->batch * 4)};
     for (const Range &r : others)
@@ -246,7 +259,7 @@ mb_status mb_scan_prefill_ckpt(const mb_scan_args *args, float *h_last, float *h
     if (h_last && !aligned16(h_last)) return MB_ERR_INVALID_ARG;
     const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
     const int64_t tok = chans * args->seqlen * es;
-    const int64_t bc = args->batch * args->seqlen * args->d_state * es;
+    const int64_t bc = bc_bytes(args);
     const Range rc = range_of(h_ckpt, ck_bytes);
     const Range others[] = {range_of(args->x, tok), range_of(args->z, tok), range_of(args->dt, tok),
                             range_of(args->B, bc), range_of(args->C, bc), range_of(args->y, tok),
@@ -283,7 +296,7 @@ mb_status mb_scan_backward(const mb_scan_args *args, const float *h_ckpt, const 
     for (const void *q : al)
         if (q && !aligned16(q)) return MB_ERR_INVALID_ARG;
     const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
-    const int64_t tok = chans * L * es, bcb = Bn * L * N * es, st_b = chans * N * 4;
+    const int64_t tok = chans * L * es, bcb = bc_bytes(args), st_b = chans * N * 4;
     const int64_t nchunks = (L + mbscan::kCkptSteps - 1) / mbscan::kCkptSteps;
     // outputs: disjoint from each other and from every input
     const Range outs[] = {range_of(g.dx, any_tokens ? tok : 0), range_of(g.ddt, any_tokens ? tok : 0),
@@ -322,8 +335,9 @@ mb_status mb_scan_backward(const mb_scan_args *args, const float *h_ckpt, const 
 
 mb_status mb_rmsnorm(const void *add, float *residual, const float *w, float eps, void *out,
                      int64_t batch, int64_t width, int32_t dtype, void *stream) {
-    if (batch < 0 || width < 0 || batch > kMaxTokens || width > 8192 || width % 8 != 0)
-        return width > 8192 || width % 8 != 0 ? MB_ERR_UNSUPPORTED : MB_ERR_INVALID_ARG;
+    if (batch < 0 || width < 0 || batch > kMaxTokens || width > kMaxTokens) return MB_ERR_INVALID_ARG;
+    if (width % 8 != 0) return MB_ERR_UNSUPPORTED;
+    if (batch > 0 && width > 0 && batch > kMaxTokens / width) return MB_ERR_INVALID_ARG;
     if (dtype != MB_F32 && dtype != MB_BF16) return MB_ERR_INVALID_ARG;
     if (batch * width == 0) return MB_OK;
     if (!(eps >= 0.f)) return MB_ERR_INVALID_ARG;

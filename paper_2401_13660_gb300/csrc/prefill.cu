@@ -368,12 +368,14 @@ __global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant
 // ---------------------------------------------------------------------------
 // Host side: tensor maps and the launch.
 
-// [batch, L, inner] tensor with a (box_inner x kT x 1) box.
+// [batch, L, inner] tensor with a (box_inner x kT x 1) box; rows (b, t) are
+// `row` elements apart (row >= inner).
 bool make_map(CUtensorMap *m, const void *base, bool bf16, int64_t batch, int64_t L, int64_t inner,
-              int box_inner) {
+              int box_inner, int64_t row = 0) {
     const int64_t es = bf16 ? 2 : 4;
+    if (row == 0) row = inner;
     const uint64_t dims[3] = {(uint64_t)inner, (uint64_t)L, (uint64_t)batch};
-    const uint64_t strides[2] = {(uint64_t)(inner * es), (uint64_t)(L * inner * es)};
+    const uint64_t strides[2] = {(uint64_t)(row * es), (uint64_t)(L * row * es)};
     const uint32_t box[3] = {(uint32_t)box_inner, (uint32_t)kT, 1};
     return encode_tmap(m, base, (int)es, 3, dims, strides, box);
 }
@@ -389,8 +391,8 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
     if (!make_map(&a.tm_dt, p.dt, bf16, p.batch, p.seqlen, p.d_inner, kCh) ||
         !make_map(&a.tm_x, p.x, bf16, p.batch, p.seqlen, p.d_inner, kCh) ||
         (p.z && !make_map(&a.tm_z, p.z, bf16, p.batch, p.seqlen, p.d_inner, kCh)) ||
-        !make_map(&a.tm_B, p.B, bf16, p.batch, p.seqlen, kDState, kDState) ||
-        !make_map(&a.tm_C, p.C, bf16, p.batch, p.seqlen, kDState, kDState) ||
+        !make_map(&a.tm_B, p.B, bf16, p.batch, p.seqlen, kDState, kDState, p.bc_stride) ||
+        !make_map(&a.tm_C, p.C, bf16, p.batch, p.seqlen, kDState, kDState, p.bc_stride) ||
         !make_map(&a.tm_y, p.y, bf16, p.batch, p.seqlen, p.d_inner, kCh))
         return cudaErrorInvalidValue;
     const size_t smem = sizeof(Smem<T, kCh, STAGES>) + 128;

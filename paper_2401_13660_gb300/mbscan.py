@@ -35,7 +35,7 @@ class mb_scan_args(ctypes.Structure):
     _fields_ = [
         ("batch", ctypes.c_int64), ("seqlen", ctypes.c_int64),
         ("d_inner", ctypes.c_int64), ("d_state", ctypes.c_int64),
-        ("dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("dtype", ctypes.c_int32), ("bc_stride", ctypes.c_int32),
         ("x", ctypes.c_void_p), ("z", ctypes.c_void_p), ("dt", ctypes.c_void_p),
         ("B", ctypes.c_void_p), ("C", ctypes.c_void_p),
         ("A", ctypes.c_void_p), ("D", ctypes.c_void_p), ("dt_bias", ctypes.c_void_p),
@@ -117,10 +117,35 @@ def _need(t, name, dtype=None, shape=None, device=None):
         raise ValueError(f"{name} is on {t.device}, expected {device}")
 
 
+def _bc_row_stride(B, C, batch, L, N, dtype, dev):
+    """Row stride (elements) shared by B and C [batch, L, N]: N for
+    contiguous tensors, or S when both are column blocks of wider rows
+    (strides (L*S, S, 1))."""
+    strides = set()
+    for name, t in (("B", B), ("C", C)):
+        if not isinstance(t, torch.Tensor):
+            raise TypeError(f"{name} must be a torch.Tensor")
+        if t.dtype != dtype or tuple(t.shape) != (batch, L, N) or t.device != dev:
+            raise ValueError(f"{name}: {t.dtype} {tuple(t.shape)} on {t.device}, expected {dtype} "
+                             f"{(batch, L, N)} on {dev}")
+        if t.is_contiguous():
+            strides.add(N)
+            continue
+        sb, st, sn = t.stride()
+        if sn != 1 or (L > 1 and sb != L * st) or st < N:
+            raise ValueError(f"{name} must be contiguous or have strides (L*S, S, 1)")
+        strides.add(st if L > 1 or batch == 1 else sb)
+    if len(strides) != 1:
+        raise ValueError("B and C must share one row stride")
+    return strides.pop()
+
+
 def make_args(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None) -> mb_scan_args:
     """Fill mb_scan_args from tensors. x, dt, z, y: [batch, L, d_inner];
-    B, C: [batch, L, d_state] (all one dtype, fp32 or bf16); A: [d_inner,
-    d_state], D, dt_bias: [d_inner], h0: [batch, d_inner, d_state] (fp32)."""
+    B, C: [batch, L, d_state] (all one dtype, fp32 or bf16), contiguous or
+    column blocks of wider rows (strides (L*S, S, 1): bc_stride = S); A:
+    [d_inner, d_state], D, dt_bias: [d_inner], h0: [batch, d_inner, d_state]
+    (fp32)."""
     if x.dtype not in _DTYPES:
         raise TypeError(f"unsupported input dtype {x.dtype}")
     batch, L, Dn = x.shape
@@ -128,8 +153,7 @@ def make_args(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None) -> mb
     dev = x.device
     for name, t in (("x", x), ("dt", dt), ("z", z), ("y", y)):
         _need(t, name, x.dtype, (batch, L, Dn), dev)
-    for name, t in (("B", B), ("C", C)):
-        _need(t, name, x.dtype, (batch, L, N), dev)
+    S = _bc_row_stride(B, C, batch, L, N, x.dtype, dev)
     _need(A, "A", torch.float32, (Dn, N), dev)
     _need(D, "D", torch.float32, (Dn,), dev)
     _need(dt_bias, "dt_bias", torch.float32, (Dn,), dev)
@@ -137,6 +161,7 @@ def make_args(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None) -> mb
     a = mb_scan_args()
     a.batch, a.seqlen, a.d_inner, a.d_state = batch, L, Dn, N
     a.dtype = _DTYPES[x.dtype]
+    a.bc_stride = 0 if S == N else S
     a.x, a.z, a.dt, a.B, a.C = (t.data_ptr() if t is not None else None for t in (x, z, dt, B, C))
     a.A, a.D, a.dt_bias, a.h0 = (t.data_ptr() if t is not None else None for t in (A, D, dt_bias, h0))
     a.y = y.data_ptr()

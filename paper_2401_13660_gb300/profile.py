@@ -46,13 +46,18 @@ def algorithmic_bytes(entry: str, w, s_in: int) -> int:
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--entry", choices=["prefill", "verify", "rollback", "step", "backward"], required=True)
-    ap.add_argument("--workload", required=True, choices=sorted(WORKLOADS))
+    ap.add_argument("--entry", choices=["prefill", "verify", "rollback", "step", "backward", "decode_model"],
+                    required=True)
+    ap.add_argument("--workload", required=True,
+                    help="a workload of inputs.WORKLOADS, or for --entry decode_model a decoder.CONFIGS name")
+    ap.add_argument("--batch", type=int, default=256, help="streams of --entry decode_model")
     ap.add_argument("--iters", type=int, default=5)
     ap.add_argument("--layers", type=int, default=4, help="state sets cycled by --entry step")
     a = ap.parse_args()
-    w = WORKLOADS[a.workload]
     dev = torch.device("cuda:0")
+    if a.entry == "decode_model":
+        return decode_model(a, dev)
+    w = WORKLOADS[a.workload]
     mb.load_library()
     nsets = a.layers if a.entry == "step" else 1
     sets = []
@@ -125,6 +130,28 @@ def main():
     nbytes = algorithmic_bytes(a.entry, w, 2 if w.dtype == "bf16" else 4)
     print(json.dumps({"entry": a.entry, "workload": w.name, "iters": a.iters, "us_per_launch": round(us, 3),
                       "algorithmic_bytes": nbytes, "GB/s": round(nbytes / (us * 1e-6) / 1e9, 1)}))
+
+
+def decode_model(a, dev):
+    """Whole-model decoding: capture the step's CUDA graph, replay it."""
+    from .decoder import CONFIGS, Decoder
+
+    dec = Decoder(CONFIGS[a.workload], batch=a.batch, device=dev, seed=1)
+    dec.capture()
+    tok = torch.randint(0, 256, (a.batch,), device=dev, generator=torch.Generator(device=dev).manual_seed(8))
+    dec.step(tok)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    ev[0].record()
+    for _ in range(a.iters):
+        dec.step(tok)
+    ev[1].record()
+    torch.cuda.synchronize()
+    ms = ev[0].elapsed_time(ev[1]) / max(a.iters, 1)
+    nb = dec.bytes_per_step()
+    print(json.dumps({"entry": "decode_model", "workload": a.workload, "batch": a.batch, "iters": a.iters,
+                      "ms_per_step": round(ms, 4), "bytes_per_step": nb, "GB/s": round(nb / ms / 1e6, 1),
+                      "generated_bytes_per_s": round(a.batch / (ms * 1e-3), 1)}))
 
 
 if __name__ == "__main__":

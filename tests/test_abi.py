@@ -200,7 +200,7 @@ def test_block_kernel_checks():
     f = ctypes.c_float(1e-5)
     assert lib.mb_rmsnorm(add, res, w, f, out, 4, 64, mb.MB_BF16, None) in (mb.MB_OK, mb.MB_ERR_CUDA)
     assert lib.mb_rmsnorm(add, res, w, f, out, 4, 60, mb.MB_BF16, None) == mb.MB_ERR_UNSUPPORTED
-    assert lib.mb_rmsnorm(add, res, w, f, out, 4, 8200, mb.MB_BF16, None) == mb.MB_ERR_UNSUPPORTED
+    assert lib.mb_rmsnorm(add, res, w, f, out, 4, 8200, mb.MB_BF16, None) in (mb.MB_OK, mb.MB_ERR_CUDA)
     assert lib.mb_rmsnorm(add, res, w, f, res + 64, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
     assert lib.mb_rmsnorm(add, res, w, ctypes.c_float(-1.0), out, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
     assert lib.mb_rmsnorm(add, None, w, f, out, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
@@ -210,6 +210,17 @@ def test_block_kernel_checks():
     assert lib.mb_conv1d_step(x, x + 32, cw, cb, co, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
     assert lib.mb_conv1d_step(x, st, None, cb, co, 4, 64, mb.MB_BF16, None) == mb.MB_ERR_INVALID_ARG
     assert lib.mb_conv1d_step(x, st, cw, cb, co, 0, 64, mb.MB_BF16, None) == mb.MB_OK
+
+
+def test_bc_stride_checks():
+    a = _args(L=4)
+    a.bc_stride = 12                                    # < d_state
+    assert _prefill(a) == mb.MB_ERR_INVALID_ARG
+    a.bc_stride = 20                                    # 40 bytes: not a multiple of 16 for bf16
+    assert _prefill(a) == mb.MB_ERR_INVALID_ARG
+    a = _args(L=4, dtype=mb.MB_F32)
+    a.bc_stride = 20                                    # 80 bytes: fine for fp32
+    assert _prefill(a) in (mb.MB_OK, mb.MB_ERR_CUDA)
 
 
 def test_binding_rejects_cpu_shape_errors():

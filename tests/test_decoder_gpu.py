@@ -19,7 +19,7 @@ DT = {"f32": torch.float32, "bf16": torch.bfloat16}
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("batch, width, with_add", [(4, 64, True), (256, 2304, True), (3, 8192, False),
-                                                     (1, 8, True)])
+                                                     (1, 8, True), (9, 12296, True)])
 def test_rmsnorm_matches_oracle(dtype, batch, width, with_add):
     g = torch.Generator(device=DEV).manual_seed(width)
     res = torch.randn(batch, width, device=DEV, generator=g)
@@ -34,7 +34,7 @@ def test_rmsnorm_matches_oracle(dtype, batch, width, with_add):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-@pytest.mark.parametrize("batch, width", [(4, 64), (256, 4608), (3, 8)])
+@pytest.mark.parametrize("batch, width", [(4, 64), (256, 4608), (3, 8), (7, 136)])
 def test_conv_step_matches_oracle(dtype, batch, width):
     g = torch.Generator(device=DEV).manual_seed(batch + width)
     state = torch.zeros(batch, 3, width, device=DEV, dtype=DT[dtype])
