@@ -55,6 +55,9 @@ constexpr int kThreads = 32 * kWarps;
 constexpr int kPrefillLanesPerChannel = MB_PREFILL_LPC;
 constexpr int kPrefillStages = 4;  // TMA ring depth for long spans
 constexpr int kVerifyStages = 2;   // verify spans are short
+#ifndef MB_VERIFY_MINB
+#define MB_VERIFY_MINB 8   // verify CTAs per SM the register budget must allow (64 registers)
+#endif
 
 // Lane geometry: LPC lanes share one channel, each holding kSPL states.
 template <int LPC>
@@ -188,7 +191,8 @@ __device__ __forceinline__ float reduce_steps(const float (&part)[LPC], int q) {
 }
 
 template <typename T, int LPC, int STAGES, bool kStoreAll, bool kCkpt>
-__global__ void __launch_bounds__(kThreads) prefill_kernel(const __grid_constant__ PrefillArgs a) {
+__global__ void __launch_bounds__(kThreads, kStoreAll ? MB_VERIFY_MINB : 1)
+    prefill_kernel(const __grid_constant__ PrefillArgs a) {
     using G = Geom<LPC>;
     constexpr int CH = G::kCh;
     using S = Smem<T, CH, STAGES>;
@@ -434,6 +438,9 @@ cudaError_t launch_prefill_ckpt(const ScanParams &p, bool bf16, cudaStream_t s) 
 cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s) {
     if (p.batch == 0 || p.d_inner == 0 || p.seqlen == 0) return cudaSuccess;
     constexpr int LPC = kPrefillLanesPerChannel;
+    if (p.seqlen <= kT)   // one chunk: a single ring stage suffices (smaller CTAs, more resident)
+        return bf16 ? launch_typed<__nv_bfloat16, LPC, 1, true>(p, s)
+                    : launch_typed<float, LPC, 1, true>(p, s);
     return bf16 ? launch_typed<__nv_bfloat16, LPC, kVerifyStages, true>(p, s)
                 : launch_typed<float, LPC, kVerifyStages, true>(p, s);
 }
