@@ -107,7 +107,10 @@ __global__ void __launch_bounds__(1024) rmsnorm_kernel(const T *__restrict__ add
 }
 
 constexpr int kConvThreads = 256;
-constexpr int kConvRows = 4;   // batch rows per thread (the weights are loaded once for them)
+#ifndef MB_CONV_ROWS
+#define MB_CONV_ROWS 4
+#endif
+constexpr int kConvRows = MB_CONV_ROWS;   // batch rows per thread (the weights are loaded once for them)
 
 // One decode step of the causal depthwise convolution (kernel 4) and SiLU:
 //   out[b,d] = silu(sum_{j<3} w[d,j] state[b,j,d] + w[d,3] x[b,d] + bias[d]),

@@ -187,6 +187,26 @@ def test_verify_matches_prefill_and_oracle_small(dtype):
     torch.testing.assert_close(h_all[:, -1], hl, rtol=1e-5, atol=1e-6)
 
 
+@pytest.mark.parametrize("dtype,L", [("bf16", 5), ("f32", 16), ("bf16", 1)])
+def test_verify_single_chunk_ragged_stays_in_bounds(dtype, L):
+    """Spans of at most one chunk stage the per-position states in shared
+    memory and write them with one tile store per CTA: positions past L and
+    channels past d_inner (536 = 16 full 32-channel tiles + 24) must be clipped,
+    so a sentinel tail after h_all stays untouched and every stream's rows
+    match the oracle."""
+    b, D = 3, 8 * 67
+    inp = make_inputs(b, L, D, 16, dtype, "normal", seed=33, device=DEV)
+    n = b * L * D * 16
+    big = torch.full((n + 8192,), float("nan"), device=DEV)
+    h_all = big[:n].view(b, L, D, 16)
+    y = torch.empty_like(inp["x"])
+    mb.mb_scan_verify(inp["x"], inp["dt"], inp["B"], inp["C"], inp["A"], y, h_all, z=inp.get("z"),
+                      D=inp.get("D"), dt_bias=inp.get("dt_bias"), h0=inp.get("h0"))
+    ry, _, rall = oracle_scan(inp, want_h_all=True)
+    assert torch.isnan(big[n:]).all()
+    assert rel_err(y, ry) <= TOL[dtype] and rel_err(h_all, rall) <= TOL[dtype]
+
+
 def test_rollback_edges_and_alias():
     inp = make_inputs(6, 16, 32, 16, "f32", "normal", seed=41, device=DEV)
     _, h_all = _verify(inp)
