@@ -108,7 +108,7 @@ __global__ void __launch_bounds__(1024) rmsnorm_kernel(const T *__restrict__ add
 
 constexpr int kConvThreads = 256;
 #ifndef MB_CONV_ROWS
-#define MB_CONV_ROWS 4
+#define MB_CONV_ROWS 2
 #endif
 constexpr int kConvRows = MB_CONV_ROWS;   // batch rows per thread (the weights are loaded once for them)
 
