@@ -70,6 +70,22 @@ typedef enum { MB_F32 = 0, MB_BF16 = 1 } mb_dtype;
  *   dt_bias  : [d_inner] fp32 added to dt before softplus; NULL means 0
  *   h0       : [batch, d_inner, d_state] fp32 initial state; NULL means 0
  *   y        : [batch, seqlen, d_inner], dtype, output
+ * Fused low-rank Delta projection (Eq. 3: Delta = softplus(W_Delta (W_R x)),
+ * W_Delta of size d_inner x r). Leave dt_low NULL to pass dt itself. When
+ * dt_low is not NULL, dt must be NULL and the kernels evaluate
+ *     dt[b,t,d] = sum_{k < dt_rank} dt_low[b,t,k] * W_dt[d,k]
+ * in fp32 on the tensor cores (bf16 operands, fp32 accumulation; dt is never
+ * rounded to the input dtype):
+ *   dt_low   : [batch, seqlen, dt_rank], dtype (W_R x); row (b, t) starts
+ *              dt_low_stride elements after row (b, t-1), e.g. the first
+ *              dt_rank columns of the [dt_low | B | C] x-projection output
+ *   W_dt     : [d_inner, dt_rank], dtype, contiguous (W_Delta)
+ *   dt_rank  : r; supported: dtype MB_BF16, r % 16 == 0, 64 <= r <= 256
+ *              (MB_ERR_UNSUPPORTED otherwise)
+ *   dt_low_stride: 0 means dt_rank; otherwise >= dt_rank, a multiple of 8
+ * Accepted by mb_scan_prefill and mb_scan_verify; mb_step, mb_step_resume,
+ * mb_scan_prefill_ckpt and mb_scan_backward return MB_ERR_UNSUPPORTED (they
+ * take dt).
  */
 typedef struct {
     int64_t batch, seqlen, d_inner, d_state;
@@ -82,6 +98,10 @@ typedef struct {
     const float *dt_bias;
     const float *h0;
     void *y;
+    const void *dt_low;
+    const void *W_dt;
+    int32_t dt_rank;
+    int32_t dt_low_stride;
 } mb_scan_args;
 
 /* Bytes of device workspace that mb_scan_prefill / mb_scan_verify need for

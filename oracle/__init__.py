@@ -10,6 +10,8 @@ Functions (MambaByte, Eq. 2-3, discretisation appendix, Table 6, Algorithm 1):
 
 * ``scan``     - the layer core over a whole span: y, final state, and
                  optionally every per-position state (verify).
+* ``delta_projection`` - the pre-softplus timestep of Eq. 3 from its low-rank
+                 factor: W_Delta (W_R x), as an fp64 matrix product.
 * ``step``     - one recurrent decode step (a scan of length 1).
 * ``rollback`` - keep the state after ``accept`` drafted bytes.
 * ``accept_topk`` - Algorithm 1's bifurcation: leading drafted bytes whose
@@ -147,6 +149,16 @@ def scan_backward(x, dt, B, C, A, dout, *, z=None, D=None, dt_bias=None, h0=None
     if rc != 0:
         raise RuntimeError(f"oracle_scan_backward failed ({rc})")
     return g
+
+
+def delta_projection(dt_low, W_dt):
+    """Eq. 3: the timestep before softplus is W_Delta applied to the rank-r
+    projection W_R x. dt_low [batch, L, r] holds W_R x, W_dt [d_inner, r] is
+    W_Delta; returns dt [batch, L, d_inner] = sum_k dt_low[..., k] W_dt[d, k],
+    in fp64."""
+    dl = np.asarray(dt_low, dtype=np.float64)
+    w = np.asarray(W_dt, dtype=np.float64)
+    return np.matmul(dl, w.T)
 
 
 def step(state, x, dt, B, C, A, *, z=None, D=None, dt_bias=None, b_rule=B_EULER, nthreads=None):

@@ -26,7 +26,15 @@ struct ScanParams {
     float *h_out;      // prefill: h_last (may be null); verify: h_all; step: state
     StatusBlock *status;
     float *h_ckpt;     // prefill with checkpoints: state before every kCkptSteps-step chunk
+    // Fused low-rank Delta projection (Eq. 3): when dt_low is set (dt is then
+    // null), dt[b, t, d] = sum_k dt_low[b, t, k] * W_dt[d, k], k < dt_rank.
+    const void *dt_low;        // [batch, seqlen, dt_rank], rows dt_low_stride elements apart (bf16)
+    const void *W_dt;          // [d_inner, dt_rank] (bf16)
+    int64_t dt_rank, dt_low_stride;
 };
+
+constexpr int kRankTile = 64;    // dt_rank elements per 128-byte swizzled TMA box
+constexpr int kMaxRank = 256;
 
 constexpr int kDState = 16;
 constexpr int kCkptSteps = 16;   // steps between the state checkpoints of the training forward
@@ -34,8 +42,12 @@ constexpr int kCkptSteps = 16;   // steps between the state checkpoints of the t
 // Encode a tiled TMA tensor map over `base` (bf16 when elem_bytes == 2, else
 // fp32): dims innermost first, strides[i] = byte stride of dimension i + 1,
 // box = tile extent per dimension. Out-of-range elements load as zeros.
+// swizzle: 0 (rows stored as they are), 64 or 128: rows of the box (that
+// many bytes) stored with that swizzle, 16-byte chunk j of row i at chunk
+// j ^ (i % 8) for 128 (destination 1024-byte aligned), j ^ ((i / 2) % 4) for
+// 64 (destination 512-byte aligned).
 bool encode_tmap(CUtensorMap *m, const void *base, int elem_bytes, int rank, const uint64_t *dims,
-                 const uint64_t *strides, const uint32_t *box);
+                 const uint64_t *strides, const uint32_t *box, int swizzle = 0);
 
 // Launchers: return the cudaError_t of the launch.
 cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s);

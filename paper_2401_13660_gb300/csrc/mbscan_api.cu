@@ -39,6 +39,30 @@ int64_t bc_bytes(const mb_scan_args *a) {
     return ((rows - 1) * stride + a->d_state) * es;
 }
 
+// Bytes spanned by dt_low (fused Delta projection): rows dt_low_stride apart.
+int64_t dtl_bytes(const mb_scan_args *a) {
+    const int64_t rows = a->batch * a->seqlen;
+    if (!a->dt_low || rows <= 0) return 0;
+    const int64_t stride = a->dt_low_stride ? a->dt_low_stride : a->dt_rank;
+    return ((rows - 1) * stride + a->dt_rank) * 2;
+}
+int64_t wdt_bytes(const mb_scan_args *a) { return a->dt_low ? a->d_inner * a->dt_rank * 2 : 0; }
+
+// The fused Delta projection's arguments (dt_low set); MB_OK when dt_low is null.
+mb_status check_fused(const mb_scan_args *a) {
+    if (!a->dt_low) return MB_OK;
+    if (a->dt) return MB_ERR_INVALID_ARG;
+    if (a->dt_rank <= 0 || a->dt_low_stride < 0) return MB_ERR_INVALID_ARG;
+    if (a->dtype != MB_BF16 || a->dt_rank % 16 != 0 || a->dt_rank < mbscan::kRankTile ||
+        a->dt_rank > mbscan::kMaxRank)
+        return MB_ERR_UNSUPPORTED;
+    if (a->dt_low_stride != 0 && (a->dt_low_stride < a->dt_rank || a->dt_low_stride % 8 != 0))
+        return MB_ERR_INVALID_ARG;
+    if (a->batch * a->d_inner > 0 && !a->W_dt) return MB_ERR_INVALID_ARG;
+    if (!aligned16(a->dt_low) || (a->W_dt && !aligned16(a->W_dt))) return MB_ERR_INVALID_ARG;
+    return MB_OK;
+}
+
 // Validate the common part of a scan problem; `need_seqlen1` for mb_step.
 mb_status check_args(const mb_scan_args *a, bool need_seqlen1, bool need_y = true) {
     if (a == nullptr) return MB_ERR_INVALID_ARG;
@@ -52,12 +76,14 @@ mb_status check_args(const mb_scan_args *a, bool need_seqlen1, bool need_y = tru
     if (a->d_inner % 8 != 0) return MB_ERR_UNSUPPORTED;
     if (a->batch > kMaxTokens || a->seqlen > kMaxTokens || a->d_inner > kMaxTokens)
         return MB_ERR_INVALID_ARG;
+    if (mb_status f = check_fused(a); f != MB_OK) return f;
     const int64_t chans = a->batch * a->d_inner;
     if (a->seqlen > 0 && chans > kMaxTokens / a->seqlen) return MB_ERR_INVALID_ARG;
     if (chans > kMaxTokens / mbscan::kDState) return MB_ERR_INVALID_ARG;
     const bool any_tokens = a->batch * a->seqlen * a->d_inner > 0;
     const bool any_chan = chans > 0;
-    if (any_tokens && (!a->x || !a->dt || !a->B || !a->C || (need_y && !a->y))) return MB_ERR_INVALID_ARG;
+    if (any_tokens && (!a->x || !(a->dt || a->dt_low) || !a->B || !a->C || (need_y && !a->y)))
+        return MB_ERR_INVALID_ARG;
     if (any_chan && !a->A) return MB_ERR_INVALID_ARG;
     const void *ptrs[] = {a->x, a->z, a->dt, a->B, a->C, a->A, a->D, a->dt_bias, a->h0, a->y};
     for (const void *p : ptrs)
@@ -71,7 +97,8 @@ mb_status check_args(const mb_scan_args *a, bool need_seqlen1, bool need_y = tru
                          range_of(a->B, bc), range_of(a->C, bc),
                          range_of(a->A, a->d_inner * a->d_state * 4),
                          range_of(a->D, a->d_inner * 4), range_of(a->dt_bias, a->d_inner * 4),
-                         range_of(a->h0, chans * a->d_state * 4)};
+                         range_of(a->h0, chans * a->d_state * 4),
+                         range_of(a->dt_low, dtl_bytes(a)), range_of(a->W_dt, wdt_bytes(a))};
     for (const Range &r : ins)
         if (overlap(ry, r)) return MB_ERR_INVALID_ARG;
     return MB_OK;
@@ -89,6 +116,10 @@ ScanParams to_params(const mb_scan_args *a, float *h_out, StatusBlock *status) {
     p.h_out = h_out;
     p.status = status;
     p.h_ckpt = nullptr;
+    p.dt_low = a->dt_low;
+    p.W_dt = a->W_dt;
+    p.dt_rank = a->dt_low ? a->dt_rank : 0;
+    p.dt_low_stride = a->dt_low ? (a->dt_low_stride ? a->dt_low_stride : a->dt_rank) : 0;
     return p;
 }
 
@@ -125,7 +156,9 @@ mb_status mb_scan_prefill(const mb_scan_args *args, float *h_last, void *ws, siz
         const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
         const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
         if (overlap(rh, range_of(args->y, tok)) || overlap(rh, range_of(args->x, tok)) ||
-            overlap(rh, range_of(args->dt, tok)) || overlap(rh, range_of(args->z, tok)))
+            overlap(rh, range_of(args->dt, tok)) || overlap(rh, range_of(args->z, tok)) ||
+            overlap(rh, range_of(args->dt_low, dtl_bytes(args))) ||
+            overlap(rh, range_of(args->W_dt, wdt_bytes(args))))
             return MB_ERR_INVALID_ARG;
     }
     if (args->batch * args->d_inner == 0) return MB_OK;
@@ -146,7 +179,9 @@ mb_status mb_scan_verify(const mb_scan_args *args, float *h_all, void *ws, size_
         const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
         if (overlap(ra, range_of(args->h0, args->batch * args->d_inner * args->d_state * 4)) ||
             overlap(ra, range_of(args->y, tok)) || overlap(ra, range_of(args->x, tok)) ||
-            overlap(ra, range_of(args->dt, tok)) || overlap(ra, range_of(args->z, tok)))
+            overlap(ra, range_of(args->dt, tok)) || overlap(ra, range_of(args->z, tok)) ||
+            overlap(ra, range_of(args->dt_low, dtl_bytes(args))) ||
+            overlap(ra, range_of(args->W_dt, wdt_bytes(args))))
             return MB_ERR_INVALID_ARG;
     }
     if (n_all == 0) return MB_OK;
@@ -196,6 +231,7 @@ mb_status mb_accept_topk(const void *logits, int32_t dtype, const uint8_t *draft
 mb_status mb_step(const mb_scan_args *args, float *state, void *stream) {
     mb_status st = check_args(args, true);
     if (st != MB_OK) return st;
+    if (args->dt_low) return MB_ERR_UNSUPPORTED;   // the step kernel takes dt
     const int64_t chans = args->batch * args->d_inner;
     if (chans == 0) return MB_OK;
     if (state == nullptr || !aligned16(state)) return MB_ERR_INVALID_ARG;
@@ -205,7 +241,8 @@ mb_status mb_step(const mb_scan_args *args, float *state, void *stream) {
     const Range others[] = {range_of(args->y, tok), range_of(args->x, tok), range_of(args->z, tok),
                             range_of(args->dt, tok), range_of(args->B, bc_bytes(args)),
                             range_of(args->C, bc_bytes(args)),
-                            range_of(args->A, args->d_inner * args->d_state * 4)};
+                            range_of(args->A, args->d_inner * args->d_state * 4),
+                            range_of(args->dt_low, dtl_bytes(args)), range_of(args->W_dt, wdt_bytes(args))};
     for (const Range &r : others)
         if (overlap(rs, r)) return MB_ERR_INVALID_ARG;
     ScanParams p = to_params(args, state, nullptr);
@@ -217,6 +254,7 @@ mb_status mb_step_resume(const mb_scan_args *args, const float *h_all, const int
                          int64_t k, float *state, void *ws, size_t ws_bytes, void *stream) {
     mb_status st = check_args(args, true);
     if (st != MB_OK) return st;
+    if (args->dt_low) return MB_ERR_UNSUPPORTED;   // the step kernel takes dt
     const int64_t chans = args->batch * args->d_inner;
     if (k < 1 || k > kMaxTokens) return MB_ERR_INVALID_ARG;
     if (chans > 0 && k > kMaxTokens * 16 / (chans * args->d_state)) return MB_ERR_INVALID_ARG;
@@ -234,7 +272,8 @@ mb_status mb_step_resume(const mb_scan_args *args, const float *h_all, const int
                             range_of(args->dt, tok), range_of(args->B, bc_bytes(args)),
                             range_of(args->C, bc_bytes(args)),
                             range_of(args->A, args->d_inner * args->d_state * 4),
-                            range_of(h_all, args->batch * k * per), range_of(accept, args->batch * 4)};
+                            range_of(h_all, args->batch * k * per), range_of(accept, args->batch * 4),
+                            range_of(args->dt_low, dtl_bytes(args)), range_of(args->W_dt, wdt_bytes(args))};
     for (const Range &r : others)
         if (overlap(rs, r)) return MB_ERR_INVALID_ARG;
     if (args->h0 && args->h0 != state && overlap(rs, range_of(args->h0, args->batch * per)))
@@ -251,6 +290,7 @@ mb_status mb_scan_prefill_ckpt(const mb_scan_args *args, float *h_last, float *h
                                size_t ws_bytes, void *stream) {
     mb_status st = check_args(args, false);
     if (st != MB_OK) return st;
+    if (args->dt_low) return MB_ERR_UNSUPPORTED;   // the training path takes dt
     if ((st = check_ws(args, ws, ws_bytes)) != MB_OK) return st;
     const int64_t chans = args->batch * args->d_inner;
     const int64_t nchunks = (args->seqlen + mbscan::kCkptSteps - 1) / mbscan::kCkptSteps;
@@ -281,6 +321,7 @@ mb_status mb_scan_backward(const mb_scan_args *args, const float *h_ckpt, const 
                            size_t ws_bytes, void *stream) {
     mb_status st = check_args(args, false, false);
     if (st != MB_OK) return st;
+    if (args->dt_low) return MB_ERR_UNSUPPORTED;   // the training path takes dt
     if (!grads) return MB_ERR_INVALID_ARG;
     if ((st = check_ws(args, ws, ws_bytes)) != MB_OK) return st;
     const int64_t Bn = args->batch, L = args->seqlen, Dn = args->d_inner, N = args->d_state;

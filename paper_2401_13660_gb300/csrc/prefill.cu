@@ -54,9 +54,15 @@ constexpr int kThreads = 32 * kWarps;
 #endif
 constexpr int kPrefillLanesPerChannel = MB_PREFILL_LPC;
 constexpr int kPrefillStages = 4;  // TMA ring depth for long spans
+// With the fused Delta projection and dt_rank > 64 each stage also holds two
+// or more dt_low boxes: one stage less keeps 4 CTAs per SM.
+constexpr int kPrefillStagesWide = 3;
 constexpr int kVerifyStages = 2;   // verify spans are short
 #ifndef MB_VERIFY_MINB
 #define MB_VERIFY_MINB 8   // verify CTAs per SM the register budget must allow (64 registers)
+#endif
+#ifndef MB_VERIFY_FUSED_MINB
+#define MB_VERIFY_FUSED_MINB 6   // the same with the Delta projection in the kernel (80 registers)
 #endif
 
 // Lane geometry: LPC lanes share one channel, each holding kSPL states.
@@ -68,13 +74,13 @@ struct Geom {
     static constexpr int kCh = kWarps * kChPerWarp;  // channels per CTA
 };
 
-template <typename T, int CH>
-struct Raw {  // TMA destinations; every member offset is a multiple of 128 B
-    T dt[kT][CH];
+template <typename T, int CH, bool kFuse>
+struct alignas(128) Raw {  // TMA destinations; every member offset is a multiple of 128 B
     T x[kT][CH];
     T z[kT][CH];
     T B[kT][kDState];
     T C[kT][kDState];
+    T dt[kFuse ? 1 : kT][CH];   // unused when Delta is projected in the kernel
 };
 
 template <int CH>
@@ -83,9 +89,9 @@ struct Conv {
     float2 xs[kT][CH];          // (D*x, silu(z)); silu(z) = 1 without a gate
 };
 
-template <typename T, int CH, int STAGES>
+template <typename T, int CH, int STAGES, bool kFuse>
 struct Smem {
-    Raw<T, CH> raw[STAGES];
+    Raw<T, CH, kFuse> raw[STAGES];
     Conv<CH> cv[2];
     T ys[2][kT][CH];            // output tiles, written out by TMA stores
     uint64_t full[STAGES];
@@ -93,20 +99,46 @@ struct Smem {
 
 struct PrefillArgs {
     CUtensorMap tm_dt, tm_x, tm_z, tm_B, tm_C, tm_y;
+    // fused Delta projection: dt_low [batch, L, r] and W_dt [D, r] in 64-wide,
+    // 128-byte-swizzled boxes (kRankTile columns x kT rows, resp. x CH rows)
+    CUtensorMap tm_dtl, tm_wdt;
     ScanParams p;
     int has_gate;
+    int nbox;      // ceil(dt_rank / kRankTile)
 };
 
-template <typename T, int CH, int STAGES>
-__device__ __forceinline__ void issue_chunk(Smem<T, CH, STAGES> &s, const PrefillArgs &a, int stage,
-                                            int64_t chunk, int d0, int b) {
+// Shared-memory layout of the fused Delta projection, after the Smem struct:
+// per stage nbox dt_low boxes (kT x 128 B), then the CTA's W_dt slice
+// (nbox boxes of CH x 128 B); 1024-byte aligned for the 128-byte swizzle.
+constexpr uint32_t kDtlBox = kT * 128;
+template <int CH>
+struct FuseLayout {
+    static constexpr uint32_t kWBox = CH * 128;
+    static uint32_t bytes(int stages, int nbox) { return 1024 + (uint32_t)nbox * (stages * kDtlBox + kWBox); }
+};
+
+// Byte offset of 16-byte chunk `chunk` of row `row` in a 128-byte-swizzled box.
+__device__ __forceinline__ uint32_t swz(int row, int chunk) {
+    return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
+template <typename T, int CH, int STAGES, bool kFuse>
+__device__ __forceinline__ void issue_chunk(Smem<T, CH, STAGES, kFuse> &s, const PrefillArgs &a, int stage,
+                                            int64_t chunk, int d0, int b, unsigned char *fz,
+                                            uint32_t extra_bytes = 0) {
     constexpr uint32_t tok = kT * CH * sizeof(T), bc = kT * kDState * sizeof(T);
-    const uint32_t bytes = (a.has_gate ? 3 : 2) * tok + 2 * bc;
+    const uint32_t bytes = (a.has_gate ? 2 : 1) * tok + 2 * bc + extra_bytes +
+                           (kFuse ? (uint32_t)a.nbox * kDtlBox : tok);
     uint64_t *bar = &s.full[stage];
     mbar_arrive_expect_tx(bar, bytes);
     const int t = (int)(chunk * kT);
-    Raw<T, CH> &r = s.raw[stage];
-    tma_load_3d(&r.dt[0][0], &a.tm_dt, bar, d0, t, b);
+    Raw<T, CH, kFuse> &r = s.raw[stage];
+    if constexpr (kFuse) {
+        for (int bx = 0; bx < a.nbox; ++bx)
+            tma_load_3d(fz + (stage * a.nbox + bx) * kDtlBox, &a.tm_dtl, bar, bx * kRankTile, t, b);
+    } else {
+        tma_load_3d(&r.dt[0][0], &a.tm_dt, bar, d0, t, b);
+    }
     tma_load_3d(&r.x[0][0], &a.tm_x, bar, d0, t, b);
     if (a.has_gate) tma_load_3d(&r.z[0][0], &a.tm_z, bar, d0, t, b);
     tma_load_3d(&r.B[0][0], &a.tm_B, bar, 0, t, b);
@@ -129,7 +161,9 @@ __device__ __forceinline__ float4 ld_quad(const __nv_bfloat16 *p) {
 }
 
 // Per-thread constants of the conversion role: thread converts the adjacent
-// channel pair (2 cp, 2 cp + 1) at steps th, th + kRows, ...
+// channel pair (2 cp, 2 cp + 1) at steps th, th + kRows, ... With the fused
+// Delta projection the pairs follow the mma accumulator layout: warp w owns
+// channels 8w .. 8w+7, lane l the pair 4w + l % 4 at steps l / 4 and l / 4 + 8.
 template <int CH>
 struct ConvRole {
     static constexpr int kPairsPerRow = CH / 2;
@@ -140,10 +174,41 @@ struct ConvRole {
     bool ok;
 };
 
+// Delta before softplus for the fused projection (Eq. 3, W_Delta (W_R x)):
+// warp w multiplies the chunk's dt_low tile [kT x r] by its 8 channels' W_dt
+// rows [8 x r]^T on the tensor cores, r / 16 mma steps; both operands come
+// from 128-byte-swizzled TMA boxes (dtl: this stage's dt_low boxes, w: the
+// CTA's W_dt boxes). acc[0..1]: steps lane / 4, channels 8w + 2 (lane % 4) + {0, 1};
+// acc[2..3]: the same channels at step lane / 4 + 8.
+template <int CH>
+__device__ __forceinline__ void project_delta(float (&acc)[4], uint32_t dtl, uint32_t w, int nks) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const uint32_t tok = order_token();   // the operands are valid from here (after the stage's wait)
+    dtl += tok;
+    w += tok;
+    acc[0] = acc[1] = acc[2] = acc[3] = 0.f;
+    const int arow = lane & 15, achunk = lane >> 4;             // A: 4 matrices (rows 0-7 / 8-15, k 0-7 / 8-15)
+    const int brow = 8 * warp + (lane & 7), bchunk = (lane >> 3) & 1;   // B: 2 matrices (k 0-7 / 8-15)
+    for (int ks = 0; ks < nks; ++ks) {
+        const int bx = ks >> 2, c0 = (ks & 3) * 2;
+        uint32_t a[4], b[2];
+        ldsm_x4(dtl + bx * kDtlBox + swz(arow, c0 + achunk), a);
+        ldsm_x2(w + bx * FuseLayout<CH>::kWBox + swz(brow, c0 + bchunk), b);
+        mma_bf16_16816(acc, a, b);
+    }
+}
+
+struct FuseCtx {
+    uint32_t dtl, w;   // shared addresses: this stage's dt_low boxes, the W_dt boxes
+    int nks;           // dt_rank / 16
+};
+
 // Convert one chunk: raw TMA tiles -> fp32 (Delta, Delta*x), (D*x, silu z).
-template <typename T, int CH>
-__device__ __forceinline__ void convert(Conv<CH> &cv, const Raw<T, CH> &r, const ConvRole<CH> &cr,
-                                        int64_t t0, int64_t L, bool gate) {
+template <typename T, int CH, bool kFuse>
+__device__ __forceinline__ void convert(Conv<CH> &cv, const Raw<T, CH, kFuse> &r, const ConvRole<CH> &cr,
+                                        int64_t t0, int64_t L, bool gate, const FuseCtx &fx) {
+    float acc[4];
+    if constexpr (kFuse) project_delta<CH>(acc, fx.dtl, fx.w, fx.nks);
 #pragma unroll
     for (int k = 0; k < ConvRole<CH>::kPasses; ++k) {
         const int t = cr.th + ConvRole<CH>::kRows * k;
@@ -151,7 +216,9 @@ __device__ __forceinline__ void convert(Conv<CH> &cv, const Raw<T, CH> &r, const
         float4 dg = make_float4(0.f, 0.f, 0.f, 0.f), xs = make_float4(0.f, 1.f, 0.f, 1.f);
         if (cr.ok && t0 + t < L) {
             const float2 xv = ld_pair(&r.x[t][c]);
-            const float2 dv = ld_pair(&r.dt[t][c]);
+            float2 dv;
+            if constexpr (kFuse) dv = make_float2(acc[2 * k], acc[2 * k + 1]);
+            else dv = ld_pair(&r.dt[t][c]);
             const float d0 = softplus(dv.x + cr.bias.x), d1 = softplus(dv.y + cr.bias.y);
             dg = make_float4(d0, d0 * xv.x, d1, d1 * xv.y);
             xs.x = cr.dsk.x * xv.x;
@@ -190,15 +257,28 @@ __device__ __forceinline__ float reduce_steps(const float (&part)[LPC], int q) {
     }
 }
 
-template <typename T, int LPC, int STAGES, bool kStoreAll, bool kCkpt>
-__global__ void __launch_bounds__(kThreads, kStoreAll ? MB_VERIFY_MINB : 1)
+template <typename T, int LPC, int STAGES, bool kStoreAll, bool kCkpt, bool kFuse>
+__global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED_MINB : MB_VERIFY_MINB) : 1)
     prefill_kernel(const __grid_constant__ PrefillArgs a) {
     using G = Geom<LPC>;
     constexpr int CH = G::kCh;
-    using S = Smem<T, CH, STAGES>;
+    static_assert(!kFuse || (LPC == 4 && sizeof(T) == 2 && CH == 8 * kWarps),
+                  "the fused Delta projection maps one 8-channel mma tile per warp (bf16)");
+    using S = Smem<T, CH, STAGES, kFuse>;
     extern __shared__ unsigned char smem_dyn[];
     S &s = *reinterpret_cast<S *>((reinterpret_cast<uintptr_t>(smem_dyn) + 127) &
                                   ~static_cast<uintptr_t>(127));
+    // fused Delta projection: dt_low stage boxes, then the W_dt boxes (1024-aligned)
+    uint32_t fz_addr = 0;   // shared address of the first dt_low box
+    unsigned char *fz = nullptr;
+    FuseCtx fx{0u, 0u, 0};
+    if constexpr (kFuse) {
+        const uint32_t sbase = smem_u32(smem_dyn);
+        fz_addr = (sbase + 128 + (uint32_t)sizeof(S) + 1023u) & ~1023u;
+        fz = smem_dyn + (fz_addr - sbase);
+        fx.w = fz_addr + (uint32_t)(STAGES * a.nbox) * kDtlBox;
+        fx.nks = (int)(a.p.dt_rank / 16);
+    }
     const ScanParams &p = a.p;
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
@@ -216,13 +296,27 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? MB_VERIFY_MINB : 1)
     }
     __syncthreads();
     if (tid == 0) {
-        for (int st = 0; st < STAGES && st < nchunks; ++st) issue_chunk(s, a, st, st, d0, b);
+        for (int st = 0; st < STAGES && st < nchunks; ++st) {
+            // the CTA's W_dt slice rides on chunk 0's barrier (its bytes are
+            // part of that arrival's expected count)
+            const bool wslice = kFuse && st == 0;
+            issue_chunk(s, a, st, st, d0, b, fz, wslice ? (uint32_t)a.nbox * FuseLayout<CH>::kWBox : 0u);
+            if (wslice)
+                for (int bx = 0; bx < a.nbox; ++bx)
+                    tma_load_2d(fz + (uint32_t)(STAGES * a.nbox) * kDtlBox + (uint32_t)bx * FuseLayout<CH>::kWBox,
+                                &a.tm_wdt, &s.full[0], bx * kRankTile, d0);
+        }
     }
 
     // ---- conversion role
     ConvRole<CH> cr;
-    cr.cp = tid % ConvRole<CH>::kPairsPerRow;
-    cr.th = tid / ConvRole<CH>::kPairsPerRow;
+    if constexpr (kFuse) {
+        cr.cp = 4 * warp + (lane & 3);
+        cr.th = lane >> 2;
+    } else {
+        cr.cp = tid % ConvRole<CH>::kPairsPerRow;
+        cr.th = tid / ConvRole<CH>::kPairsPerRow;
+    }
     {
         const int64_t dc = d0 + 2 * cr.cp;   // D % 8 == 0: both channels valid or neither
         cr.ok = dc < D;
@@ -252,7 +346,13 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? MB_VERIFY_MINB : 1)
 
     // ---- prologue: chunk 0
     bool ok = nchunks > 0 ? mbar_wait(&s.full[0], 0) : true;
-    if (ok && nchunks > 0) convert(s.cv[0], s.raw[0], cr, 0, L, gate);
+    if constexpr (kFuse) ok = __all_sync(kFull, ok);   // mma.sync needs the whole warp
+    auto stage_fx = [&](int st) {   // the fused projection's operands for ring stage st
+        FuseCtx f = fx;
+        if constexpr (kFuse) f.dtl = fz_addr + (uint32_t)(st * a.nbox) * kDtlBox;
+        return f;
+    };
+    if (ok && nchunks > 0) convert(s.cv[0], s.raw[0], cr, 0, L, gate, stage_fx(0));
     if (__syncthreads_or(ok ? 0 : 1)) {
         if (tid == 0) {
             report(p.status, 4 /* MB_ERR_TIMEOUT */, 0);
@@ -267,7 +367,8 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? MB_VERIFY_MINB : 1)
         // (1) chunk i+1: wait for its tiles and convert them
         const int nst = (int)((i + 1) % STAGES);
         ok = has_next ? mbar_wait(&s.full[nst], (uint32_t)(((i + 1) / STAGES) & 1)) : true;
-        if (has_next && ok) convert(s.cv[(i + 1) & 1], s.raw[nst], cr, t0 + kT, L, gate);
+        if constexpr (kFuse) ok = __all_sync(kFull, ok);
+        if (has_next && ok) convert(s.cv[(i + 1) & 1], s.raw[nst], cr, t0 + kT, L, gate, stage_fx(nst));
 
         // (2) chunk i: decays of all kT steps, recurrence, shares of C.h
         if constexpr (kCkpt) {   // state before chunk i, for the backward's recompute
@@ -281,7 +382,7 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? MB_VERIFY_MINB : 1)
             }
         }
         const Conv<CH> &cv = s.cv[i & 1];
-        const Raw<T, CH> &rs = s.raw[i % STAGES];   // B, C straight from the TMA tile
+        const Raw<T, CH, kFuse> &rs = s.raw[i % STAGES];   // B, C straight from the TMA tile
         float2 ab[kT][G::kPairs];
         float gx[kT];
 #pragma unroll
@@ -356,7 +457,7 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? MB_VERIFY_MINB : 1)
             // now) is free: refill it with chunk i + STAGES
             if (i + STAGES < nchunks) {
                 fence_proxy_async_smem();
-                issue_chunk(s, a, (int)(i % STAGES), i + STAGES, d0, b);
+                issue_chunk(s, a, (int)(i % STAGES), i + STAGES, d0, b, fz);
             }
         }
     }
@@ -384,7 +485,7 @@ bool make_map(CUtensorMap *m, const void *base, bool bf16, int64_t batch, int64_
     return encode_tmap(m, base, (int)es, 3, dims, strides, box);
 }
 
-template <typename T, int LPC, int STAGES, bool kStoreAll, bool kCkpt = false>
+template <typename T, int LPC, int STAGES, bool kStoreAll, bool kCkpt = false, bool kFuse = false>
 cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
     constexpr int kCh = Geom<LPC>::kCh;
     const bool bf16 = sizeof(T) == 2;
@@ -392,15 +493,32 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
     memset(&a, 0, sizeof(a));
     a.p = p;
     a.has_gate = p.z != nullptr;
-    if (!make_map(&a.tm_dt, p.dt, bf16, p.batch, p.seqlen, p.d_inner, kCh) ||
-        !make_map(&a.tm_x, p.x, bf16, p.batch, p.seqlen, p.d_inner, kCh) ||
+    size_t fuse_bytes = 0;
+    if constexpr (kFuse) {
+        // dt_low [batch, L, r] (rows dt_low_stride apart) and W_dt [D, r], both
+        // in kRankTile-wide boxes with the 128-byte swizzle; columns past r read 0
+        a.nbox = (int)((p.dt_rank + kRankTile - 1) / kRankTile);
+        const uint64_t ldims[3] = {(uint64_t)p.dt_rank, (uint64_t)p.seqlen, (uint64_t)p.batch};
+        const uint64_t lstr[2] = {(uint64_t)p.dt_low_stride * 2, (uint64_t)(p.seqlen * p.dt_low_stride) * 2};
+        const uint32_t lbox[3] = {kRankTile, kT, 1};
+        const uint64_t wdims[2] = {(uint64_t)p.dt_rank, (uint64_t)p.d_inner};
+        const uint64_t wstr[1] = {(uint64_t)p.dt_rank * 2};
+        const uint32_t wbox[2] = {kRankTile, (uint32_t)kCh};
+        if (!encode_tmap(&a.tm_dtl, p.dt_low, 2, 3, ldims, lstr, lbox, 128) ||
+            !encode_tmap(&a.tm_wdt, p.W_dt, 2, 2, wdims, wstr, wbox, 128))
+            return cudaErrorInvalidValue;
+        fuse_bytes = FuseLayout<kCh>::bytes(STAGES, a.nbox);
+    } else {
+        if (!make_map(&a.tm_dt, p.dt, bf16, p.batch, p.seqlen, p.d_inner, kCh)) return cudaErrorInvalidValue;
+    }
+    if (!make_map(&a.tm_x, p.x, bf16, p.batch, p.seqlen, p.d_inner, kCh) ||
         (p.z && !make_map(&a.tm_z, p.z, bf16, p.batch, p.seqlen, p.d_inner, kCh)) ||
         !make_map(&a.tm_B, p.B, bf16, p.batch, p.seqlen, kDState, kDState, p.bc_stride) ||
         !make_map(&a.tm_C, p.C, bf16, p.batch, p.seqlen, kDState, kDState, p.bc_stride) ||
         !make_map(&a.tm_y, p.y, bf16, p.batch, p.seqlen, p.d_inner, kCh))
         return cudaErrorInvalidValue;
-    const size_t smem = sizeof(Smem<T, kCh, STAGES>) + 128;
-    auto k = prefill_kernel<T, LPC, STAGES, kStoreAll, kCkpt>;
+    const size_t smem = sizeof(Smem<T, kCh, STAGES, kFuse>) + 128 + fuse_bytes;
+    auto k = prefill_kernel<T, LPC, STAGES, kStoreAll, kCkpt, kFuse>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const dim3 grid((unsigned)(((p.d_inner + kCh - 1) / kCh) * p.batch));
@@ -423,6 +541,10 @@ cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s) {
         return cudaMemsetAsync(p.h_out, 0, bytes, s);
     }
     constexpr int LPC = kPrefillLanesPerChannel;
+    if (p.dt_low)   // fused Delta projection (bf16 only; the API checks)
+        return !bf16 ? cudaErrorInvalidValue
+               : p.dt_rank <= kRankTile ? launch_typed<__nv_bfloat16, LPC, kPrefillStages, false, false, true>(p, s)
+                                        : launch_typed<__nv_bfloat16, LPC, kPrefillStagesWide, false, false, true>(p, s);
     return bf16 ? launch_typed<__nv_bfloat16, LPC, kPrefillStages, false>(p, s)
                 : launch_typed<float, LPC, kPrefillStages, false>(p, s);
 }
@@ -438,6 +560,11 @@ cudaError_t launch_prefill_ckpt(const ScanParams &p, bool bf16, cudaStream_t s) 
 cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s) {
     if (p.batch == 0 || p.d_inner == 0 || p.seqlen == 0) return cudaSuccess;
     constexpr int LPC = kPrefillLanesPerChannel;
+    if (p.dt_low) {   // fused Delta projection (bf16 only; the API checks)
+        if (!bf16) return cudaErrorInvalidValue;
+        return p.seqlen <= kT ? launch_typed<__nv_bfloat16, LPC, 1, true, false, true>(p, s)
+                              : launch_typed<__nv_bfloat16, LPC, kVerifyStages, true, false, true>(p, s);
+    }
     if (p.seqlen <= kT)   // one chunk: a single ring stage suffices (smaller CTAs, more resident)
         return bf16 ? launch_typed<__nv_bfloat16, LPC, 1, true>(p, s)
                     : launch_typed<float, LPC, 1, true>(p, s);

@@ -108,6 +108,42 @@ __device__ __forceinline__ void bulk_wait_read_all() {
 // Wait until every committed bulk store has completed.
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
+// ---- warp-level tensor-core pieces (mma.sync) for small in-kernel
+// contractions. ldmatrix: four (two) 8x8 16-bit matrices from shared memory;
+// lanes 8j .. 8j+7 give the row addresses of matrix j, and lane l receives
+// row l / 4, columns 2 (l % 4) and 2 (l % 4) + 1 of every matrix, one 32-bit
+// register per matrix (lower column in the low half).
+// These are plain (non-volatile) asm so that the compiler may interleave them
+// with independent work. They are ordered after the wait that makes their
+// shared-memory operand valid only through their address: derive it from
+// order_token(), which is produced after that wait.
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+    asm("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+        : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t (&r)[2]) {
+    asm("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
+}
+// A zero the compiler cannot see through, emitted in program order (volatile):
+// adding it to an address makes the load depend on everything before it.
+__device__ __forceinline__ uint32_t order_token() {
+    uint32_t z;
+    asm volatile("mov.u32 %0, 0;" : "=r"(z)::"memory");
+    return z;
+}
+// d += A B for one 16 x 8 x 16 tile: A row-major 16 x 16 bf16 (registers:
+// rows g, g+8 at columns 2t.., then the same rows at columns 8+2t.., where
+// g = lane / 4, t = lane % 4), B column-major 16 x 8 bf16 (rows 2t.. and
+// 8+2t.. of column g), d fp32 (rows g and g+8, columns 2t and 2t+1).
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+        "{%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
 // ---- packed fp32 pairs: one FFMA2 / FMUL2 / FADD2 instruction per two lanes
 // of math (the sm_100 float2 builtins).
 __device__ __forceinline__ float2 mul2(float2 a, float2 b) { return __fmul2_rn(a, b); }

@@ -30,7 +30,8 @@ EncodeTiledFn encode_fn() {
 }  // namespace
 
 bool encode_tmap(CUtensorMap *m, const void *base, int elem_bytes, int rank, const uint64_t *dims,
-                 const uint64_t *strides, const uint32_t *box) {
+                 const uint64_t *strides, const uint32_t *box, int swizzle) {
+    if (swizzle != 0 && swizzle != 64 && swizzle != 128) return false;
     EncodeTiledFn enc = encode_fn();
     if (!enc || rank < 1 || rank > 5) return false;
     cuuint64_t d[5], st[4];
@@ -44,7 +45,9 @@ bool encode_tmap(CUtensorMap *m, const void *base, int elem_bytes, int rank, con
     const CUtensorMapDataType dt = elem_bytes == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16
                                                    : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
     return enc(m, dt, (cuuint32_t)rank, const_cast<void *>(base), d, st, bx, es,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+               CU_TENSOR_MAP_INTERLEAVE_NONE,
+               swizzle == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                              : (swizzle == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_NONE),
                CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 

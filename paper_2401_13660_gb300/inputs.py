@@ -17,6 +17,9 @@ workload is bf16):
 * A[d, n] = -(n + 1) (S4D-real initialisation of Mamba's diagonal A)
 * h0 = 0, or ~ N(0, 0.1^2) for workloads that resume from a cached state
 * accept (verify workloads) ~ uniform integers in [0, seqlen]
+* fused Delta projection (dt_rank r > 0, drawn last): dt_low ~ N(0, 1)
+  [batch, L, r] and W_dt ~ N(0, 1/r) [d_inner, r], so that dt_low W_dt^T is
+  again ~ N(0, 1); dt itself is then dropped (the kernels form it)
 """
 from __future__ import annotations
 
@@ -39,6 +42,7 @@ class Workload:
     seed: int
     layers: int = 1       # distinct state/input sets (decode step over a layer stack)
     accept: bool = False  # draw per-stream accept counts (speculative verify)
+    dt_rank: int = 0      # > 0: dt comes as the low-rank pair (dt_low, W_dt) of Eq. 3
     note: str = field(default="", compare=False)
 
 
@@ -55,6 +59,12 @@ WORKLOADS = {
                  note="speculative verify of a 16-byte drafted span on 32 streams"),
         Workload("step_b256_D4608_x48", 256, 1, 4608, 16, "bf16", "normal", 4, layers=48,
                  note="MambaByte-1.6B (d=2304, e=2) batched decode step, 48 layers"),
+        Workload("mambabyte353m_prefill_fused_r64_b8_L8192", 8, 8192, 2048, 16, "bf16", "zeros", 5,
+                 dt_rank=64, note="MambaByte-353M layer prefill, Delta projection (r = d/16) in the kernel"),
+        Workload("mambabyte972m_prefill_fused_r112_b4_L8192", 4, 8192, 3584, 16, "bf16", "normal", 6,
+                 dt_rank=112, note="MambaByte-972M layer prefill, Delta projection (r = d/16) in the kernel"),
+        Workload("verify_fused_r64_s32_k16_D2048", 32, 16, 2048, 16, "bf16", "normal", 7, accept=True,
+                 dt_rank=64, note="speculative verify (353M layer), Delta projection in the kernel"),
     ]
 }
 
@@ -71,12 +81,14 @@ def _normal(gen, shape, device, std=1.0):
 
 def make_inputs(batch: int, seqlen: int, d_inner: int, d_state: int, dtype: str = "bf16",
                 h0: str = "zeros", seed: int = 0, device="cpu", accept: bool = False,
-                gate: bool = True) -> dict:
+                gate: bool = True, dt_rank: int = 0) -> dict:
     """Draw one problem. Returns a dict of contiguous torch tensors on `device`.
 
     Keys: x, z (None if gate=False), dt, B, C (input dtype); A [d_inner, d_state],
     D [d_inner], dt_bias [d_inner] (fp32); h0 [batch, d_inner, d_state] fp32 or
-    None; accept [batch] int32 (only if accept=True).
+    None; accept [batch] int32 (only if accept=True). With dt_rank > 0, dt is
+    None and dt_low [batch, L, dt_rank], W_dt [d_inner, dt_rank] (input dtype)
+    are given instead.
     """
     device = torch.device(device)
     gen = torch.Generator(device=device)
@@ -103,10 +115,14 @@ def make_inputs(batch: int, seqlen: int, d_inner: int, d_state: int, dtype: str 
     if accept:
         out["accept"] = torch.randint(0, seqlen + 1, (batch,), generator=gen, device=device,
                                       dtype=torch.int64).to(torch.int32)
+    if dt_rank > 0:
+        out["dt_low"] = _normal(gen, (batch, seqlen, dt_rank), device).to(td)
+        out["W_dt"] = _normal(gen, (d_inner, dt_rank), device, std=1.0 / math.sqrt(dt_rank)).to(td)
+        out["dt"] = None
     return out
 
 
 def workload_inputs(w: Workload, device="cpu", layer: int = 0) -> dict:
     """Inputs of one layer of a workload (layer > 0 reseeds so layers differ)."""
     return make_inputs(w.batch, w.seqlen, w.d_inner, w.d_state, w.dtype, w.h0,
-                       seed=w.seed * 1000 + layer, device=device, accept=w.accept)
+                       seed=w.seed * 1000 + layer, device=device, accept=w.accept, dt_rank=w.dt_rank)

@@ -40,6 +40,8 @@ class mb_scan_args(ctypes.Structure):
         ("B", ctypes.c_void_p), ("C", ctypes.c_void_p),
         ("A", ctypes.c_void_p), ("D", ctypes.c_void_p), ("dt_bias", ctypes.c_void_p),
         ("h0", ctypes.c_void_p), ("y", ctypes.c_void_p),
+        ("dt_low", ctypes.c_void_p), ("W_dt", ctypes.c_void_p),
+        ("dt_rank", ctypes.c_int32), ("dt_low_stride", ctypes.c_int32),
     ]
 
 
@@ -117,40 +119,50 @@ def _need(t, name, dtype=None, shape=None, device=None):
         raise ValueError(f"{name} is on {t.device}, expected {device}")
 
 
+def _row_stride(name, t, batch, L, width, dtype, dev):
+    """Row stride (elements) of t [batch, L, width]: width when contiguous,
+    or S when t is a column block of wider rows (strides (L*S, S, 1))."""
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype or tuple(t.shape) != (batch, L, width) or t.device != dev:
+        raise ValueError(f"{name}: {t.dtype} {tuple(t.shape)} on {t.device}, expected {dtype} "
+                         f"{(batch, L, width)} on {dev}")
+    if t.is_contiguous():
+        return width
+    sb, st, sn = t.stride()
+    if sn != 1 or (L > 1 and sb != L * st) or st < width:
+        raise ValueError(f"{name} must be contiguous or have strides (L*S, S, 1)")
+    return st if L > 1 or batch == 1 else sb
+
+
 def _bc_row_stride(B, C, batch, L, N, dtype, dev):
     """Row stride (elements) shared by B and C [batch, L, N]: N for
     contiguous tensors, or S when both are column blocks of wider rows
     (strides (L*S, S, 1))."""
-    strides = set()
-    for name, t in (("B", B), ("C", C)):
-        if not isinstance(t, torch.Tensor):
-            raise TypeError(f"{name} must be a torch.Tensor")
-        if t.dtype != dtype or tuple(t.shape) != (batch, L, N) or t.device != dev:
-            raise ValueError(f"{name}: {t.dtype} {tuple(t.shape)} on {t.device}, expected {dtype} "
-                             f"{(batch, L, N)} on {dev}")
-        if t.is_contiguous():
-            strides.add(N)
-            continue
-        sb, st, sn = t.stride()
-        if sn != 1 or (L > 1 and sb != L * st) or st < N:
-            raise ValueError(f"{name} must be contiguous or have strides (L*S, S, 1)")
-        strides.add(st if L > 1 or batch == 1 else sb)
+    strides = {_row_stride(name, t, batch, L, N, dtype, dev) for name, t in (("B", B), ("C", C))}
     if len(strides) != 1:
         raise ValueError("B and C must share one row stride")
     return strides.pop()
 
 
-def make_args(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None) -> mb_scan_args:
+def make_args(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None, dt_low=None,
+              W_dt=None) -> mb_scan_args:
     """Fill mb_scan_args from tensors. x, dt, z, y: [batch, L, d_inner];
     B, C: [batch, L, d_state] (all one dtype, fp32 or bf16), contiguous or
     column blocks of wider rows (strides (L*S, S, 1): bc_stride = S); A:
     [d_inner, d_state], D, dt_bias: [d_inner], h0: [batch, d_inner, d_state]
-    (fp32)."""
+    (fp32). Fused Delta projection: dt = None, dt_low [batch, L, r] (contiguous
+    or a column block of wider rows) and W_dt [d_inner, r]; the kernels then
+    form dt = dt_low W_dt^T themselves."""
     if x.dtype not in _DTYPES:
         raise TypeError(f"unsupported input dtype {x.dtype}")
     batch, L, Dn = x.shape
     N = A.shape[1]
     dev = x.device
+    if (dt is None) == (dt_low is None):
+        raise ValueError("pass exactly one of dt and dt_low")
+    if dt_low is not None and W_dt is None:
+        raise ValueError("dt_low needs W_dt")
     for name, t in (("x", x), ("dt", dt), ("z", z), ("y", y)):
         _need(t, name, x.dtype, (batch, L, Dn), dev)
     S = _bc_row_stride(B, C, batch, L, N, x.dtype, dev)
@@ -162,6 +174,13 @@ def make_args(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None) -> mb
     a.batch, a.seqlen, a.d_inner, a.d_state = batch, L, Dn, N
     a.dtype = _DTYPES[x.dtype]
     a.bc_stride = 0 if S == N else S
+    if dt_low is not None:
+        r = W_dt.shape[1] if W_dt.dim() == 2 else -1
+        _need(W_dt, "W_dt", x.dtype, (Dn, r), dev)
+        S = _row_stride("dt_low", dt_low, batch, L, r, x.dtype, dev)
+        a.dt_low, a.W_dt = dt_low.data_ptr(), W_dt.data_ptr()
+        a.dt_rank = r
+        a.dt_low_stride = 0 if S == r else S
     a.x, a.z, a.dt, a.B, a.C = (t.data_ptr() if t is not None else None for t in (x, z, dt, B, C))
     a.A, a.D, a.dt_bias, a.h0 = (t.data_ptr() if t is not None else None for t in (A, D, dt_bias, h0))
     a.y = y.data_ptr()
@@ -192,9 +211,10 @@ def new_workspace(args: mb_scan_args, device) -> torch.Tensor:
 
 
 def mb_scan_prefill(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None, h_last=None,
-                    ws=None, stream=None):
-    """Prefill scan: writes y and (if given) h_last [batch, d_inner, d_state]."""
-    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0)
+                    ws=None, stream=None, dt_low=None, W_dt=None):
+    """Prefill scan: writes y and (if given) h_last [batch, d_inner, d_state].
+    dt = None with dt_low, W_dt: the fused Delta projection (see make_args)."""
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0, dt_low=dt_low, W_dt=W_dt)
     _need(h_last, "h_last", torch.float32, (a.batch, a.d_inner, a.d_state), x.device)
     if ws is None:
         ws = new_workspace(a, x.device)
@@ -205,9 +225,9 @@ def mb_scan_prefill(x, dt, B, C, A, y, *, z=None, D=None, dt_bias=None, h0=None,
 
 
 def mb_scan_verify(x, dt, B, C, A, y, h_all, *, z=None, D=None, dt_bias=None, h0=None, ws=None,
-                   stream=None):
+                   stream=None, dt_low=None, W_dt=None):
     """Verify scan of k = x.shape[1] drafted bytes: y and h_all [batch, k, d_inner, d_state]."""
-    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0)
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0, dt_low=dt_low, W_dt=W_dt)
     _need(h_all, "h_all", torch.float32, (a.batch, a.seqlen, a.d_inner, a.d_state), x.device)
     if ws is None:
         ws = new_workspace(a, x.device)
@@ -230,10 +250,11 @@ def mb_rollback(h0, h_all, accept, h_out, *, ws=None, stream=None):
     return h_out
 
 
-def mb_step(x, dt, B, C, A, y, state, *, z=None, D=None, dt_bias=None, stream=None):
+def mb_step(x, dt, B, C, A, y, state, *, z=None, D=None, dt_bias=None, stream=None, dt_low=None,
+            W_dt=None):
     """One decode step: x, dt, z, y [batch, 1, d_inner]; B, C [batch, 1, d_state];
     state [batch, d_inner, d_state] updated in place."""
-    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias)
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, dt_low=dt_low, W_dt=W_dt)
     _need(state, "state", torch.float32, (a.batch, a.d_inner, a.d_state), x.device)
     rc = load_library().mb_step(ctypes.byref(a), _ptr(state), _stream(stream))
     _check(rc, "mb_step")
@@ -241,11 +262,12 @@ def mb_step(x, dt, B, C, A, y, state, *, z=None, D=None, dt_bias=None, stream=No
 
 
 def mb_scan_prefill_ckpt(x, dt, B, C, A, y, h_ckpt=None, *, z=None, D=None, dt_bias=None, h0=None,
-                         h_last=None, ws=None, stream=None):
+                         h_last=None, ws=None, stream=None, dt_low=None, W_dt=None):
     """Training forward: prefill that also writes h_ckpt [batch, ceil(L / 16),
     d_inner, d_state], the state before every 16-step chunk (allocated when
-    None). Returns (y, h_last, h_ckpt)."""
-    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0)
+    None). Returns (y, h_last, h_ckpt). (The fused Delta projection is not
+    accepted here: MB_ERR_UNSUPPORTED.)"""
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0, dt_low=dt_low, W_dt=W_dt)
     nch = (a.seqlen + MB_CKPT_STEPS - 1) // MB_CKPT_STEPS
     if h_ckpt is None:
         h_ckpt = torch.empty(a.batch, nch, a.d_inner, a.d_state, dtype=torch.float32, device=x.device)
@@ -336,13 +358,13 @@ def mb_conv1d_step(x, state, w, out, *, bias=None, stream=None):
 
 
 def mb_step_resume(x, dt, B, C, A, y, h_all, accept, state, *, z=None, D=None, dt_bias=None, h0=None,
-                   ws=None, stream=None):
+                   ws=None, stream=None, dt_low=None, W_dt=None):
     """One decode step from the state kept after accept[s] drafted bytes:
     h0[s] (zeros if None) when accept[s] == 0, else h_all[s, accept[s]-1].
     x, dt, z, y [batch, 1, d_inner]; B, C [batch, 1, d_state]; h_all [batch,
     k, d_inner, d_state]; accept [batch] int32; state [batch, d_inner,
     d_state] is written (it may be h0 itself)."""
-    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0)
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0, dt_low=dt_low, W_dt=W_dt)
     _need(h_all, "h_all", torch.float32, None, x.device)
     if h_all.dim() != 4 or h_all.shape[0] != a.batch or tuple(h_all.shape[2:]) != (a.d_inner, a.d_state):
         raise ValueError(f"h_all: shape {tuple(h_all.shape)}, expected [batch, k, d_inner, d_state]")

@@ -27,6 +27,8 @@ def algorithmic_bytes(entry: str, w, s_in: int) -> int:
     params = D * N * 4 + 2 * D * 4
     if entry in ("prefill", "verify"):
         rd = 3 * b * L * D * s_in + 2 * b * L * N * s_in + params
+        if w.dt_rank:   # dt is formed in the kernel from dt_low [b, L, r] and W_dt [D, r]
+            rd += (b * L * w.dt_rank + D * w.dt_rank - b * L * D) * s_in
         rd += b * D * N * 4 if (w.h0 != "zeros" or entry == "verify") else 0
         wr = b * L * D * s_in + (b * D * N * 4 if entry == "prefill" else b * L * D * N * 4)
         return rd + wr
@@ -103,10 +105,11 @@ def main():
         if a.entry == "prefill":
             mb.mb_scan_prefill(s["x"], s["dt"], s["B"], s["C"], s["A"], s["y"], z=s["z"], D=s["D"],
                                dt_bias=s["dt_bias"], h0=s["h0"], h_last=s["h_last"], ws=s["ws"],
-                               stream=stream)
+                               stream=stream, dt_low=s.get("dt_low"), W_dt=s.get("W_dt"))
         elif a.entry == "verify":
             mb.mb_scan_verify(s["x"], s["dt"], s["B"], s["C"], s["A"], s["y"], s["h_all"], z=s["z"],
-                              D=s["D"], dt_bias=s["dt_bias"], h0=s["h0"], ws=s["ws"], stream=stream)
+                              D=s["D"], dt_bias=s["dt_bias"], h0=s["h0"], ws=s["ws"], stream=stream,
+                              dt_low=s.get("dt_low"), W_dt=s.get("W_dt"))
         elif a.entry == "rollback":
             mb.mb_rollback(s["h0"], s["h_all"], s["accept"], s["h_out"], ws=s["ws"], stream=stream)
         elif a.entry == "backward":

@@ -26,9 +26,16 @@ def to_np(t):
     return None if t is None else t.detach().cpu().double().numpy()
 
 
+def oracle_dt(inp):
+    """dt of an input dict: given, or formed from (dt_low, W_dt) by the oracle."""
+    if inp.get("dt") is not None:
+        return to_np(inp["dt"])
+    return oracle.delta_projection(to_np(inp["dt_low"]), to_np(inp["W_dt"]))
+
+
 def oracle_scan(inp, want_h_all=False, nthreads=None):
     """Oracle over a whole input dict from paper_2401_13660_gb300.inputs."""
-    return oracle.scan(to_np(inp["x"]), to_np(inp["dt"]), to_np(inp["B"]), to_np(inp["C"]),
+    return oracle.scan(to_np(inp["x"]), oracle_dt(inp), to_np(inp["B"]), to_np(inp["C"]),
                        to_np(inp["A"]), z=to_np(inp.get("z")), D=to_np(inp.get("D")),
                        dt_bias=to_np(inp.get("dt_bias")), h0=to_np(inp.get("h0")),
                        want_h_all=want_h_all, nthreads=nthreads)
@@ -49,6 +56,10 @@ def oracle_channels(inp, rows, chans, nthreads=None):
     h0 = inp.get("h0")
     h0s = None if h0 is None else to_np(h0.index_select(0, rows.to(h0.device))[:, chans.to(h0.device)])
     pick = lambda t: None if t is None else to_np(t[chans.to(t.device)])
-    return oracle.scan(tok(inp["x"]), tok(inp["dt"]), bc(inp["B"]), bc(inp["C"]), pick(inp["A"]),
+    if inp.get("dt") is not None:
+        dt = tok(inp["dt"])
+    else:   # fused Delta projection: the selected rows of dt_low, the selected channels of W_dt
+        dt = oracle.delta_projection(bc(inp["dt_low"]), to_np(inp["W_dt"][chans.to(inp["W_dt"].device)]))
+    return oracle.scan(tok(inp["x"]), dt, bc(inp["B"]), bc(inp["C"]), pick(inp["A"]),
                        z=tok(inp.get("z")), D=pick(inp.get("D")), dt_bias=pick(inp.get("dt_bias")),
                        h0=h0s, nthreads=nthreads)

@@ -223,6 +223,51 @@ def test_bc_stride_checks():
     assert _prefill(a) in (mb.MB_OK, mb.MB_ERR_CUDA)
 
 
+def _fused(L=4, r=64, stride=0, **kw):
+    """Arguments with the Delta projection in the kernel (dt = NULL)."""
+    a = _args(L=L, **kw)
+    a.dt = None
+    a.dt_low, a.W_dt = FAKE + (20 << 32), FAKE + (21 << 32)
+    a.dt_rank, a.dt_low_stride = r, stride
+    return a
+
+
+def test_fused_delta_checks():
+    want_launch = (mb.MB_OK, mb.MB_ERR_CUDA)             # valid: the launch then fails without a GPU
+    assert _prefill(_fused()) in want_launch
+    assert _prefill(_fused(r=144, stride=176)) in want_launch      # column block of [dt_low | B | C]
+    a = _fused()
+    a.dt = FAKE + (2 << 32)                                          # both dt and dt_low
+    assert _prefill(a) == mb.MB_ERR_INVALID_ARG
+    assert _prefill(_fused(r=48)) == mb.MB_ERR_UNSUPPORTED           # below one 64-wide box
+    assert _prefill(_fused(r=72)) == mb.MB_ERR_UNSUPPORTED           # not a multiple of 16
+    assert _prefill(_fused(r=272)) == mb.MB_ERR_UNSUPPORTED          # above 256
+    assert _prefill(_fused(dtype=mb.MB_F32)) == mb.MB_ERR_UNSUPPORTED
+    assert _prefill(_fused(r=0)) == mb.MB_ERR_INVALID_ARG
+    assert _prefill(_fused(stride=60)) == mb.MB_ERR_INVALID_ARG      # stride < rank
+    assert _prefill(_fused(r=64, stride=68)) == mb.MB_ERR_INVALID_ARG   # rows not 16-byte aligned
+    a = _fused()
+    a.W_dt = None
+    assert _prefill(a) == mb.MB_ERR_INVALID_ARG
+    a = _fused()
+    a.dt_low = a.dt_low + 8                                          # misaligned
+    assert _prefill(a) == mb.MB_ERR_INVALID_ARG
+    a = _fused()
+    a.y = a.dt_low                                                   # y overlaps dt_low
+    assert _prefill(a) == mb.MB_ERR_INVALID_ARG
+    a = _fused()
+    assert _prefill(a, h_last=a.W_dt) == mb.MB_ERR_INVALID_ARG      # h_last overlaps W_dt
+    lib = mb.load_library()
+    ws = FAKE + (200 << 32)
+    assert lib.mb_scan_prefill_ckpt(ctypes.byref(_fused(L=40)), None, FAKE + (40 << 32), ws, 256,
+                                    None) == mb.MB_ERR_UNSUPPORTED   # the training path takes dt
+    s = _fused(L=1)
+    assert _call("mb_step", s, FAKE + (210 << 32), None) == mb.MB_ERR_UNSUPPORTED   # the step takes dt
+    acc = FAKE + (220 << 32)
+    assert lib.mb_step_resume(ctypes.byref(s), FAKE + (230 << 32), acc, 4, FAKE + (210 << 32), None, 0,
+                              None) == mb.MB_ERR_UNSUPPORTED
+
+
 def test_binding_rejects_cpu_shape_errors():
     import torch
     x = torch.zeros(1, 4, 8, dtype=torch.bfloat16)
@@ -232,3 +277,13 @@ def test_binding_rejects_cpu_shape_errors():
                      torch.zeros(1, 4, 9, dtype=torch.bfloat16))
     with pytest.raises(TypeError):
         mb.make_args(x.float(), x, x, x, torch.zeros(8, 16), x)
+    B = torch.zeros(1, 4, 16, dtype=torch.bfloat16)
+    with pytest.raises(ValueError):          # neither dt nor dt_low
+        mb.make_args(x, None, B, B, torch.zeros(8, 16), x)
+    with pytest.raises(ValueError):          # both
+        mb.make_args(x, x, B, B, torch.zeros(8, 16), x, dt_low=torch.zeros(1, 4, 64, dtype=torch.bfloat16),
+                     W_dt=torch.zeros(8, 64, dtype=torch.bfloat16))
+    xdbl = torch.zeros(1, 4, 96, dtype=torch.bfloat16)
+    a = mb.make_args(x, None, xdbl[:, :, 64:80], xdbl[:, :, 80:], torch.zeros(8, 16), x,
+                     dt_low=xdbl[:, :, :64], W_dt=torch.zeros(8, 64, dtype=torch.bfloat16))
+    assert (a.dt_rank, a.dt_low_stride, a.bc_stride, a.dt) == (64, 96, 96, None)

@@ -289,3 +289,56 @@ def test_golden_fixture_and_hand_value():
     want = yssm * 1.0 / (1.0 + math.exp(-1.0))                  # z=1
     assert abs(g["y"][0][0][0] - want) < 1e-15
     assert abs(want - 0.3141092605981670) < 1e-15
+
+
+# ---------------------------------------------------------------- Delta projection (Eq. 3)
+def test_delta_projection_brute_force():
+    """dt[b,t,d] = sum_k dt_low[b,t,k] W_dt[d,k], summed here term by term in
+    plain Python on a tiny problem."""
+    rng = np.random.default_rng(7)
+    dl = rng.standard_normal((2, 3, 5))
+    w = rng.standard_normal((4, 5))
+    got = oracle.delta_projection(dl, w)
+    assert got.shape == (2, 3, 4)
+    for b in range(2):
+        for t in range(3):
+            for d in range(4):
+                want = 0.0
+                for k in range(5):
+                    want += float(dl[b, t, k]) * float(w[d, k])
+                assert abs(got[b, t, d] - want) <= 1e-12 * (1 + abs(want))
+
+
+def test_delta_projection_selects_columns_and_is_linear():
+    """One-hot rows of W_Delta pick single columns of W_R x exactly (a
+    transposed operand would pick rows instead), and the map is linear in W."""
+    rng = np.random.default_rng(8)
+    dl = rng.standard_normal((3, 4, 6))
+    pick = np.array([5, 0, 3, 3, 1, 2, 4])
+    w = np.zeros((7, 6))
+    w[np.arange(7), pick] = 1.0
+    assert np.array_equal(oracle.delta_projection(dl, w), dl[:, :, pick])
+    w1, w2 = rng.standard_normal((7, 6)), rng.standard_normal((7, 6))
+    np.testing.assert_allclose(oracle.delta_projection(dl, 2.0 * w1 - w2),
+                               2.0 * oracle.delta_projection(dl, w1) - oracle.delta_projection(dl, w2),
+                               rtol=1e-12, atol=1e-12)
+
+
+def test_scan_with_projected_delta_gated_rnn():
+    """Through the scan: with N = 1, A = -1, B = C = 1, D = 0 and no gate, the
+    recurrence is h_t = sigmoid(-v_t) h_{t-1} + softplus(v_t) x_t (the gated-RNN
+    reading of the discretisation appendix) with v_t = dt_low[t] . W_dt[d]."""
+    rng = np.random.default_rng(9)
+    L, Dn, r = 12, 3, 4
+    dl = rng.standard_normal((1, L, r))
+    w = rng.standard_normal((Dn, r)) / 2.0
+    x = rng.standard_normal((1, L, Dn))
+    ones = np.ones((1, L, 1))
+    y, hl, _ = oracle.scan(x, oracle.delta_projection(dl, w), ones, ones, -np.ones((Dn, 1)))
+    for d in range(Dn):
+        h = 0.0
+        for t in range(L):
+            v = float(dl[0, t] @ w[d])
+            h = _sig(-v) * h + math.log1p(math.exp(v)) * x[0, t, d]
+            assert abs(y[0, t, d] - h) <= 1e-12 * (1 + abs(h))
+        assert abs(hl[0, d, 0] - h) <= 1e-12 * (1 + abs(h))
