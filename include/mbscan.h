@@ -297,6 +297,20 @@ mb_status mb_conv1d_step(const void *x, void *state, const float *w, const float
 mb_status mb_check(void *ws, void *stream, int64_t *detail);
 
 /*
+ * Diagnostic of the bounded device-side waits (failure detection; an
+ * addition of this library, the paper has no counterpart). Every wait inside
+ * the kernels (for a TMA stage, a ring slot) gives up after about 2 s of SM
+ * clocks, records MB_ERR_TIMEOUT in the workspace status block and returns,
+ * so that a stalled copy cannot hang the GPU. This call runs that path on
+ * purpose: one warp waits on a barrier nothing arrives on, for wait_cycles SM
+ * clocks (1 .. 4e9), then records MB_ERR_TIMEOUT with detail = the clocks it
+ * waited. Read it with mb_check; the context stays usable.
+ *   ws, ws_bytes : a workspace as for mb_scan_prefill (>= 256 bytes, 256-byte aligned)
+ * Returns MB_ERR_INVALID_ARG for a bad workspace or wait_cycles.
+ */
+mb_status mb_selftest_timeout(void *ws, size_t ws_bytes, int64_t wait_cycles, void *stream);
+
+/*
  * mb_scan_prefill without a caller-provided workspace. (An addition of this
  * library; the paper has no counterpart.)
  *

@@ -49,7 +49,11 @@ constexpr int kCkptSteps = 16;   // steps between the state checkpoints of the t
 bool encode_tmap(CUtensorMap *m, const void *base, int elem_bytes, int rank, const uint64_t *dims,
                  const uint64_t *strides, const uint32_t *box, int swizzle = 0);
 
+constexpr long long kMaxWaitCycles = 4000000000LL;   // the kernels' wait limit (~2 s at 2 GHz)
+
 // Launchers: return the cudaError_t of the launch.
+// Bounded-wait diagnostic (selftest.cu): a wait that runs out after `limit` clocks.
+cudaError_t launch_wait_timeout(StatusBlock *sb, long long limit, cudaStream_t s);
 cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s);
 cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s);
 // Prefill that also writes p.h_ckpt [batch, ceil(L / kCkptSteps), d_inner, 16].

@@ -415,6 +415,14 @@ mb_status mb_conv1d_step(const void *x, void *state, const float *w, const float
                                               (cudaStream_t)stream));
 }
 
+mb_status mb_selftest_timeout(void *ws, size_t ws_bytes, int64_t wait_cycles, void *stream) {
+    if (ws == nullptr || ws_bytes < mbscan::kStatusBytes || (reinterpret_cast<uintptr_t>(ws) & 255u))
+        return MB_ERR_INVALID_ARG;
+    if (wait_cycles < 1 || wait_cycles > mbscan::kMaxWaitCycles) return MB_ERR_INVALID_ARG;
+    return from_cuda(mbscan::launch_wait_timeout(static_cast<StatusBlock *>(ws), (long long)wait_cycles,
+                                                 (cudaStream_t)stream));
+}
+
 mb_status mb_check(void *ws, void *stream, int64_t *detail) {
     if (detail) *detail = -1;
     if (ws == nullptr) return MB_ERR_INVALID_ARG;

@@ -82,9 +82,10 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
             lib.mb_rmsnorm.argtypes = [vp, vp, vp, ctypes.c_float, vp, i64, i64, ctypes.c_int32, vp]
             lib.mb_conv1d_step.argtypes = [vp, vp, vp, vp, vp, i64, i64, ctypes.c_int32, vp]
             lib.mb_scan_backward.argtypes = [ap, vp, vp, vp, ctypes.POINTER(mb_scan_grads), vp, sz, vp]
+            lib.mb_selftest_timeout.argtypes = [vp, sz, i64, vp]
             for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_check",
                       "mb_accept_topk", "mb_step_resume", "mb_scan_prefill_ckpt", "mb_scan_backward",
-                      "mb_rmsnorm", "mb_conv1d_step"):
+                      "mb_rmsnorm", "mb_conv1d_step", "mb_selftest_timeout"):
                 getattr(lib, f).restype = ctypes.c_int
             lib.mb_status_string.argtypes = [ctypes.c_int]
             lib.mb_status_string.restype = ctypes.c_char_p
@@ -394,6 +395,15 @@ def mb_accept_topk(logits, drafted, beta, accept=None, stream=None):
                                        int(beta), _ptr(accept), _stream(stream))
     _check(rc, "mb_accept_topk")
     return accept
+
+
+def mb_selftest_timeout(ws, wait_cycles, stream=None):
+    """Run the bounded-wait diagnostic: a kernel waits wait_cycles SM clocks on
+    a barrier nothing arrives on and records MB_ERR_TIMEOUT in ws (read it with
+    mb_check)."""
+    _need(ws, "ws", torch.uint8)
+    rc = load_library().mb_selftest_timeout(_ptr(ws), ws.numel(), int(wait_cycles), _stream(stream))
+    _check(rc, "mb_selftest_timeout")
 
 
 def mb_check(ws, stream=None):

@@ -287,3 +287,13 @@ def test_binding_rejects_cpu_shape_errors():
     a = mb.make_args(x, None, xdbl[:, :, 64:80], xdbl[:, :, 80:], torch.zeros(8, 16), x,
                      dt_low=xdbl[:, :, :64], W_dt=torch.zeros(8, 64, dtype=torch.bfloat16))
     assert (a.dt_rank, a.dt_low_stride, a.bc_stride, a.dt) == (64, 96, 96, None)
+
+
+def test_selftest_timeout_checks():
+    lib = mb.load_library()
+    ws = FAKE + (200 << 32)
+    assert lib.mb_selftest_timeout(None, 256, 1000, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_selftest_timeout(ws, 16, 1000, None) == mb.MB_ERR_INVALID_ARG        # too small
+    assert lib.mb_selftest_timeout(ws + 16, 256, 1000, None) == mb.MB_ERR_INVALID_ARG   # not 256-aligned
+    assert lib.mb_selftest_timeout(ws, 256, 0, None) == mb.MB_ERR_INVALID_ARG
+    assert lib.mb_selftest_timeout(ws, 256, 5 * 10**9, None) == mb.MB_ERR_INVALID_ARG  # above the kernels' limit
