@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "internal.h"
 
 namespace mbscan {
@@ -72,6 +74,43 @@ __device__ __forceinline__ float2 ldg2(const float *p) { return __ldg(reinterpre
 __device__ __forceinline__ float2 ldg2(const __nv_bfloat16 *p) {
     unsigned u = __ldg(reinterpret_cast<const unsigned *>(p));
     return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
+}
+
+// ---- Programmatic dependent launch. Kernels launched with launch_pdl may
+// start while the previous kernel on the stream is still draining; each such
+// kernel runs pdl_wait() before its first global-memory access, which returns
+// once every prerequisite grid has completed and its writes are visible, so
+// only shared-memory set-up overlaps the predecessor. pdl_trigger() lets the
+// next kernel launch early (it still waits for this one to complete).
+#ifndef MB_PDL
+#define MB_PDL 1
+#endif
+__device__ __forceinline__ void pdl_wait() {
+#if MB_PDL
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+#endif
+}
+__device__ __forceinline__ void pdl_trigger() {
+#if MB_PDL
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+#endif
+}
+
+// Launch `kern` on `s`, allowed to overlap the previous kernel's tail (see pdl_wait).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = MB_PDL ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
 // Record the first device-side error of a call in the workspace status block.

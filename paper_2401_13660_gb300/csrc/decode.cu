@@ -119,6 +119,8 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constan
         fence_mbar_init();
     }
     __syncthreads();
+    pdl_trigger();   // the next kernel may launch into the SMs this grid frees
+    pdl_wait();      // everything below reads or writes global memory
 
     if (warp == kStepConsumers) {
         // ---- producer
@@ -244,6 +246,8 @@ __global__ void __launch_bounds__(kRbThreads)
 rollback_kernel(const float4 *h0 /* may alias h_out */, const float4 *__restrict__ h_all,
                 const int32_t *__restrict__ accept, float4 *h_out, int64_t batch, int64_t k,
                 int64_t per_stream /* float4s */, StatusBlock *status) {
+    pdl_trigger();
+    pdl_wait();
     const int64_t i0 = ((int64_t)blockIdx.x * kRbThreads + threadIdx.x) * kRbVec;
     if (i0 >= batch * per_stream) return;
     const int64_t s = i0 / per_stream;
@@ -317,8 +321,7 @@ cudaError_t launch_step_typed(const ScanParams &p, const float *h_all, const int
         ctas = sms * (per > 0 ? per : 1);
     }
     const int grid = a.ntiles < ctas ? a.ntiles : ctas;
-    kern<<<grid, kStepThreads, smem, s>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(grid), dim3(kStepThreads), smem, s, a);
 }
 
 }  // namespace
@@ -343,10 +346,9 @@ cudaError_t launch_rollback(const float *h0, const float *h_all, const int32_t *
     const int64_t threads = batch * per / kRbVec;
     if (threads == 0) return cudaSuccess;
     const int64_t grid = (threads + kRbThreads - 1) / kRbThreads;
-    rollback_kernel<<<(unsigned)grid, kRbThreads, 0, s>>>(
-        reinterpret_cast<const float4 *>(h0), reinterpret_cast<const float4 *>(h_all), accept,
-        reinterpret_cast<float4 *>(h_out), batch, k, per, status);
-    return cudaGetLastError();
+    return launch_pdl(rollback_kernel, dim3((unsigned)grid), dim3(kRbThreads), 0, s,
+                      reinterpret_cast<const float4 *>(h0), reinterpret_cast<const float4 *>(h_all), accept,
+                      reinterpret_cast<float4 *>(h_out), batch, k, per, status);
 }
 
 }  // namespace mbscan
