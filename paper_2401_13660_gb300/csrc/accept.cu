@@ -44,7 +44,6 @@ __global__ void __launch_bounds__(32 * kAccWarps) accept_kernel(const T *__restr
     const int64_t s = blockIdx.x;
     if (threadIdx.x == 0) first_reject = (int)k;
     __syncthreads();
-    pdl_trigger();
     pdl_wait();
     for (int64_t base = 0; base < k; base += kAccWarps) {
         const int64_t i = base + warp;
@@ -75,9 +74,9 @@ cudaError_t launch_accept(const void *logits, bool bf16, const uint8_t *drafted,
     if (streams == 0) return cudaSuccess;
     const unsigned grid = (unsigned)streams;
     if (bf16)
-        return launch_pdl(accept_kernel<__nv_bfloat16>, dim3(grid), dim3(32 * kAccWarps), 0, s,
+        return launch_pdl(false, accept_kernel<__nv_bfloat16>, dim3(grid), dim3(32 * kAccWarps), 0, s,
                           static_cast<const __nv_bfloat16 *>(logits), drafted, k, beta, accept);
-    return launch_pdl(accept_kernel<float>, dim3(grid), dim3(32 * kAccWarps), 0, s,
+    return launch_pdl(false, accept_kernel<float>, dim3(grid), dim3(32 * kAccWarps), 0, s,
                       static_cast<const float *>(logits), drafted, k, beta, accept);
 }
 

@@ -220,7 +220,6 @@ __global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_con
     }
     for (int i = tid; i < kBT * 32; i += kBThreads) (&s.bc[0][0])[i] = 0.f;
     __syncthreads();
-    pdl_trigger();
     pdl_wait();   // everything below reads or writes global memory
     // ring slot j holds chunk nchunks-1-j (reverse order)
     if (tid == 0)
@@ -442,7 +441,7 @@ cudaError_t launch_backward_typed(const ScanParams &p, const GradParams &g, cuda
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const dim3 grid((unsigned)(((D + kBCh - 1) / kBCh) * Bn));
-    e = launch_pdl(k, grid, dim3(kBThreads), smem, s, a);
+    e = launch_pdl(false, k, grid, dim3(kBThreads), smem, s, a);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

@@ -62,7 +62,6 @@ __global__ void __launch_bounds__(1024) rmsnorm_kernel(const T *__restrict__ add
                                                        const float *__restrict__ w, float eps,
                                                        T *__restrict__ out, int64_t width) {
     __shared__ float red[32];
-    pdl_trigger();
     pdl_wait();
     const int64_t row = blockIdx.x;
     float *r = residual + row * width;
@@ -125,7 +124,6 @@ __global__ void __launch_bounds__(kConvThreads) conv_step_kernel(const T *__rest
                                                                  const float *__restrict__ bias,
                                                                  T *__restrict__ out, int64_t batch,
                                                                  int64_t width) {
-    pdl_trigger();
     pdl_wait();
     const int64_t groups = width / 8;
     const int64_t rowblocks = (batch + kConvRows - 1) / kConvRows;
@@ -171,10 +169,10 @@ cudaError_t launch_rmsnorm(const void *add, float *residual, const float *w, flo
     const int64_t groups = width / 8;
     const unsigned threads = (unsigned)(groups >= 1024 ? 1024 : 32 * ((groups + 31) / 32));
     if (bf16)
-        return launch_pdl(rmsnorm_kernel<__nv_bfloat16>, dim3((unsigned)batch), dim3(threads), 0, s,
+        return launch_pdl(false, rmsnorm_kernel<__nv_bfloat16>, dim3((unsigned)batch), dim3(threads), 0, s,
                           static_cast<const __nv_bfloat16 *>(add), residual, w, eps,
                           static_cast<__nv_bfloat16 *>(out), width);
-    return launch_pdl(rmsnorm_kernel<float>, dim3((unsigned)batch), dim3(threads), 0, s,
+    return launch_pdl(false, rmsnorm_kernel<float>, dim3((unsigned)batch), dim3(threads), 0, s,
                       static_cast<const float *>(add), residual, w, eps, static_cast<float *>(out), width);
 }
 
@@ -184,10 +182,10 @@ cudaError_t launch_conv_step(const void *x, void *state, const float *w, const f
     if (n == 0) return cudaSuccess;
     const unsigned grid = (unsigned)((n + kConvThreads - 1) / kConvThreads);
     if (bf16)
-        return launch_pdl(conv_step_kernel<__nv_bfloat16>, dim3(grid), dim3(kConvThreads), 0, s,
+        return launch_pdl(false, conv_step_kernel<__nv_bfloat16>, dim3(grid), dim3(kConvThreads), 0, s,
                           static_cast<const __nv_bfloat16 *>(x), static_cast<__nv_bfloat16 *>(state), w, bias,
                           static_cast<__nv_bfloat16 *>(out), batch, width);
-    return launch_pdl(conv_step_kernel<float>, dim3(grid), dim3(kConvThreads), 0, s,
+    return launch_pdl(false, conv_step_kernel<float>, dim3(grid), dim3(kConvThreads), 0, s,
                       static_cast<const float *>(x), static_cast<float *>(state), w, bias,
                       static_cast<float *>(out), batch, width);
 }

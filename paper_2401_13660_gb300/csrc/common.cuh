@@ -81,7 +81,11 @@ __device__ __forceinline__ float2 ldg2(const __nv_bfloat16 *p) {
 // kernel runs pdl_wait() before its first global-memory access, which returns
 // once every prerequisite grid has completed and its writes are visible, so
 // only shared-memory set-up overlaps the predecessor. pdl_trigger() lets the
-// next kernel launch early (it still waits for this one to complete).
+// next kernel launch before this one completes (it still waits for it). Only
+// the persistent decode step issues it: a grid of many short-lived CTAs that
+// triggers early lets the next grid's CTAs take SM slots as they free up,
+// which leaves SMs unevenly loaded when that grid fills less than every slot
+// (measured: back-to-back prefills of 448 CTAs, 822 -> 990 us).
 #ifndef MB_PDL
 #define MB_PDL 1
 #endif
@@ -96,9 +100,12 @@ __device__ __forceinline__ void pdl_trigger() {
 #endif
 }
 
-// Launch `kern` on `s`, allowed to overlap the previous kernel's tail (see pdl_wait).
+// Launch `kern` on `s`; with overlap = true it may start during the previous
+// kernel's tail (see pdl_wait). Only the decode step uses the overlap: next to
+// cuBLAS kernels (which trigger early) the short element-wise kernels measured
+// slower with it (whole-model decode 3.32 -> 3.38 ms), so they launch plainly.
 template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+cudaError_t launch_pdl(bool overlap, void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
                        Args &&...args) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
@@ -107,7 +114,7 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = MB_PDL ? 1 : 0;
+    attr[0].val.programmaticStreamSerializationAllowed = (MB_PDL && overlap) ? 1 : 0;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);

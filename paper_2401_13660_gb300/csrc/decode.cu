@@ -119,7 +119,7 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constan
         fence_mbar_init();
     }
     __syncthreads();
-    pdl_trigger();   // the next kernel may launch into the SMs this grid frees
+    pdl_trigger();   // persistent grid: the next kernel's CTAs take the SMs as this one drains
     pdl_wait();      // everything below reads or writes global memory
 
     if (warp == kStepConsumers) {
@@ -246,7 +246,6 @@ __global__ void __launch_bounds__(kRbThreads)
 rollback_kernel(const float4 *h0 /* may alias h_out */, const float4 *__restrict__ h_all,
                 const int32_t *__restrict__ accept, float4 *h_out, int64_t batch, int64_t k,
                 int64_t per_stream /* float4s */, StatusBlock *status) {
-    pdl_trigger();
     pdl_wait();
     const int64_t i0 = ((int64_t)blockIdx.x * kRbThreads + threadIdx.x) * kRbVec;
     if (i0 >= batch * per_stream) return;
@@ -321,7 +320,7 @@ cudaError_t launch_step_typed(const ScanParams &p, const float *h_all, const int
         ctas = sms * (per > 0 ? per : 1);
     }
     const int grid = a.ntiles < ctas ? a.ntiles : ctas;
-    return launch_pdl(kern, dim3(grid), dim3(kStepThreads), smem, s, a);
+    return launch_pdl(true, kern, dim3(grid), dim3(kStepThreads), smem, s, a);
 }
 
 }  // namespace
@@ -346,7 +345,7 @@ cudaError_t launch_rollback(const float *h0, const float *h_all, const int32_t *
     const int64_t threads = batch * per / kRbVec;
     if (threads == 0) return cudaSuccess;
     const int64_t grid = (threads + kRbThreads - 1) / kRbThreads;
-    return launch_pdl(rollback_kernel, dim3((unsigned)grid), dim3(kRbThreads), 0, s,
+    return launch_pdl(false, rollback_kernel, dim3((unsigned)grid), dim3(kRbThreads), 0, s,
                       reinterpret_cast<const float4 *>(h0), reinterpret_cast<const float4 *>(h_all), accept,
                       reinterpret_cast<float4 *>(h_out), batch, k, per, status);
 }

@@ -295,7 +295,6 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
         fence_mbar_init();
     }
     __syncthreads();
-    pdl_trigger();
     pdl_wait();   // everything below reads or writes global memory
     if (tid == 0) {
         for (int st = 0; st < STAGES && st < nchunks; ++st) {
@@ -524,7 +523,7 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const dim3 grid((unsigned)(((p.d_inner + kCh - 1) / kCh) * p.batch));
-    return launch_pdl(k, grid, dim3(kThreads), smem, s, a);
+    return launch_pdl(false, k, grid, dim3(kThreads), smem, s, a);
 }
 
 }  // namespace
