@@ -12,7 +12,8 @@
 // span, which the h0 / h_last interface does across calls.
 //
 // A CTA of kWarps warps owns CH = 32 kWarps / LPC channels of one batch row
-// for the whole span (small CTAs spread the channels evenly over the SMs). LPC lanes share a channel, each keeping 16 / LPC of its fp32 states in
+// for the whole span (small CTAs spread the channels evenly over the SMs).
+// LPC lanes share a channel, each keeping 16 / LPC of its fp32 states in
 // registers. The state index varies slowest across a warp, so the 8 lanes of
 // each quarter-warp read the same B, C values (a shared-memory broadcast).
 //
@@ -35,6 +36,13 @@
 //  CTA barrier per chunk orders them, after which the stage of chunk i is
 //  refilled with chunk i + STAGES.
 // Steps at or beyond L are converted with Delta = 0, which leaves h unchanged.
+//
+// Fused Delta projection (kFuse, bf16): instead of a dt tile the ring holds the
+// chunk's dt_low tile [kT x r] (W_R x of Eq. 3) and, once per CTA, the CTA's
+// W_Delta rows [CH x r], both as 128-byte-swizzled TMA boxes; in the
+// conversion step each warp forms the dt tile of its own 8 channels with r/16
+// mma.sync m16n8k16 (fp32 accumulation), and its lanes convert the channel
+// pairs and steps that the accumulator layout gives them.
 #include <string.h>
 
 #include "common.cuh"
