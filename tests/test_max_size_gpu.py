@@ -48,3 +48,28 @@ def test_step_at_the_state_limit():
     assert rel_err(state.index_select(0, r_t)[:, c_t], rh) <= TOL["bf16"]
     untouched = inp["h0"][1:].ne(state[1:]).any(dim=2).float().mean()   # every row was stepped
     assert untouched > 0.99
+
+
+def test_verify_and_rollback_beyond_32_bit_offsets():
+    b, k, Dn = 4096, 16, 4096            # h_all: 2^32 floats (16 GB)
+    inp = make_inputs(b, k, Dn, 16, "bf16", "normal", seed=93, device=DEV, accept=True)
+    y = torch.empty_like(inp["x"])
+    h_all = torch.empty(b, k, Dn, 16, device=DEV)
+    mb.mb_scan_verify(inp["x"], inp["dt"], inp["B"], inp["C"], inp["A"], y, h_all, z=inp["z"], D=inp["D"],
+                      dt_bias=inp["dt_bias"], h0=inp["h0"])
+    rows, chans = [0, 2049, b - 1], [0, 3001, Dn - 1]
+    ry, _, _ = oracle_channels(inp, rows, chans)
+    r_t, c_t = torch.tensor(rows, device=DEV), torch.tensor(chans, device=DEV)
+    assert rel_err(y.index_select(0, r_t)[:, :, c_t], ry) <= TOL["bf16"]
+    # per-position states of the last row: the oracle over its first j + 1 bytes
+    for j in (0, k - 1):
+        sub = {key: (v[:, :j + 1] if key in ("x", "z", "dt", "B", "C") else v) for key, v in inp.items()}
+        _, rh, _ = oracle_channels(sub, [b - 1], chans)
+        assert rel_err(h_all[b - 1:, j][:, c_t], rh) <= TOL["bf16"]
+    h_out = torch.empty_like(inp["h0"])
+    mb.mb_rollback(inp["h0"], h_all, inp["accept"], h_out)
+    acc = inp["accept"].long()
+    for s in rows:   # an index gather: bit-exact
+        a = int(acc[s])
+        want = inp["h0"][s] if a == 0 else h_all[s, a - 1]
+        assert torch.equal(h_out[s], want)
