@@ -137,6 +137,24 @@ mb_status mb_scan_verify(const mb_scan_args *args, float *h_all, void *ws, size_
                          void *stream);
 
 /*
+ * Verify that resumes each stream from the state kept at the previous
+ * bifurcation, with no rollback copy in between (Algorithm 1: when the
+ * corrector loop adds no byte, the next round starts from h_c, the state
+ * after the accepted drafted bytes). Stream s starts from
+ *   args->h0[s] (zeros if NULL)      if accept[s] == 0
+ *   h_all_prev[s, accept[s]-1]       if 1 <= accept[s] <= k_prev
+ * and is then scanned exactly as by mb_scan_verify (y, h_all).
+ *   h_all_prev : [batch, k_prev, d_inner, d_state] fp32, the previous
+ *                verify's per-position states (must not overlap h_all or y)
+ *   accept     : [batch] int32 on the device
+ *   ws         : required; an accept count outside [0, k_prev] is recorded
+ *                there (read it with mb_check) and that stream's y and h_all
+ *                are left untouched.
+ */
+mb_status mb_scan_verify_resume(const mb_scan_args *args, const float *h_all_prev, const int32_t *accept,
+                                int64_t k_prev, float *h_all, void *ws, size_t ws_bytes, void *stream);
+
+/*
  * Rollback at the bifurcation (Algorithm 1: the verifier resumes from the
  * state after the accepted drafted bytes). For every stream s,
  *   h_out[s] = h0[s]                 if accept[s] == 0

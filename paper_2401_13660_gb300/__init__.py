@@ -7,7 +7,7 @@ library.
 """
 _BINDING = ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_step_resume", "mb_check",
             "mb_accept_topk", "mb_scan_prefill_ckpt", "mb_scan_backward", "mb_rmsnorm", "mb_conv1d_step",
-            "mb_selftest_timeout",
+            "mb_selftest_timeout", "mb_scan_verify_resume",
             "mb_workspace_size", "mb_status_string", "mb_version", "load_library", "MbError",
             "make_args", "new_workspace")
 

@@ -31,6 +31,12 @@ struct ScanParams {
     const void *dt_low;        // [batch, seqlen, dt_rank], rows dt_low_stride elements apart (bf16)
     const void *W_dt;          // [d_inner, dt_rank] (bf16)
     int64_t dt_rank, dt_low_stride;
+    // Resume (verify after a bifurcation): when accept is set, row b starts
+    // from h0[b] (zeros if null) for accept[b] == 0, else from
+    // h_prev_all[b, accept[b] - 1] ([batch, k_prev, d_inner, 16]).
+    const float *h_prev_all;
+    const int32_t *accept;
+    int64_t k_prev;
 };
 
 constexpr int kRankTile = 64;    // dt_rank elements per 128-byte swizzled TMA box

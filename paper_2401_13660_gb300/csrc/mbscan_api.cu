@@ -120,6 +120,9 @@ ScanParams to_params(const mb_scan_args *a, float *h_out, StatusBlock *status) {
     p.W_dt = a->W_dt;
     p.dt_rank = a->dt_low ? a->dt_rank : 0;
     p.dt_low_stride = a->dt_low ? (a->dt_low_stride ? a->dt_low_stride : a->dt_rank) : 0;
+    p.h_prev_all = nullptr;
+    p.accept = nullptr;
+    p.k_prev = 0;
     return p;
 }
 
@@ -186,6 +189,37 @@ mb_status mb_scan_verify(const mb_scan_args *args, float *h_all, void *ws, size_
     }
     if (n_all == 0) return MB_OK;
     ScanParams p = to_params(args, h_all, static_cast<StatusBlock *>(ws));
+    return from_cuda(mbscan::launch_verify(p, args->dtype == MB_BF16, (cudaStream_t)stream));
+}
+
+mb_status mb_scan_verify_resume(const mb_scan_args *args, const float *h_all_prev, const int32_t *accept,
+                                int64_t k_prev, float *h_all, void *ws, size_t ws_bytes, void *stream) {
+    mb_status st = check_args(args, false);
+    if (st != MB_OK) return st;
+    if ((st = check_ws(args, ws, ws_bytes)) != MB_OK) return st;
+    if (ws == nullptr) return MB_ERR_INVALID_ARG;   // bad accept counts are reported there
+    const int64_t chans = args->batch * args->d_inner;
+    if (k_prev < 1 || k_prev > kMaxTokens) return MB_ERR_INVALID_ARG;
+    if (chans > 0 && k_prev > kMaxTokens * 16 / (chans * args->d_state)) return MB_ERR_INVALID_ARG;
+    const int64_t n_all = chans * args->seqlen * args->d_state;
+    if (n_all == 0) return MB_OK;
+    if (!h_all || !aligned16(h_all) || !h_all_prev || !aligned16(h_all_prev) || !accept ||
+        (reinterpret_cast<uintptr_t>(accept) & 3u))
+        return MB_ERR_INVALID_ARG;
+    const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
+    const int64_t tok = chans * args->seqlen * es;
+    const Range ra = range_of(h_all, n_all * 4), ry = range_of(args->y, tok);
+    const Range ins[] = {range_of(h_all_prev, chans * k_prev * args->d_state * 4),
+                         range_of(accept, args->batch * 4),
+                         range_of(args->h0, chans * args->d_state * 4), range_of(args->x, tok),
+                         range_of(args->dt, tok), range_of(args->z, tok),
+                         range_of(args->dt_low, dtl_bytes(args)), range_of(args->W_dt, wdt_bytes(args))};
+    for (const Range &r : ins)
+        if (overlap(ra, r) || overlap(ry, r)) return MB_ERR_INVALID_ARG;
+    ScanParams p = to_params(args, h_all, static_cast<StatusBlock *>(ws));
+    p.h_prev_all = h_all_prev;
+    p.accept = accept;
+    p.k_prev = k_prev;
     return from_cuda(mbscan::launch_verify(p, args->dtype == MB_BF16, (cudaStream_t)stream));
 }
 

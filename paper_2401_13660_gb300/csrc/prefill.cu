@@ -304,6 +304,17 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
     }
     __syncthreads();
     pdl_wait();   // everything below reads or writes global memory
+    // Resume: the state this row starts from (0: h0, a > 0: h_prev_all[b, a-1]).
+    // An accept count outside [0, k_prev] is reported and the row left
+    // untouched; the check comes before any copy is issued.
+    int resume_a = 0;
+    if (p.accept) {
+        resume_a = __ldg(p.accept + b);   // one batch row per CTA: uniform
+        if (resume_a < 0 || resume_a > p.k_prev) {
+            if (tid == 0 && d0 == 0) report(p.status, 1 /* MB_ERR_INVALID_ARG */, b);
+            return;
+        }
+    }
     if (tid == 0) {
         for (int st = 0; st < STAGES && st < nchunks; ++st) {
             // the CTA's W_dt slice rides on chunk 0's barrier (its bytes are
@@ -344,12 +355,15 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
     for (int k = 0; k < G::kPairs; ++k) { h[k] = make_float2(0.f, 0.f); a2[k] = h[k]; }
     if (chan_ok) {
         const float2 *Ap = reinterpret_cast<const float2 *>(p.A + d * kDState + G::kSPL * q);
-        const float2 *hp = reinterpret_cast<const float2 *>(p.h0 + ((int64_t)b * D + d) * kDState + G::kSPL * q);
+        const float *hrow = resume_a > 0
+                                ? p.h_prev_all + (((int64_t)b * p.k_prev + resume_a - 1) * D + d) * kDState
+                                : (p.h0 ? p.h0 + ((int64_t)b * D + d) * kDState : nullptr);
+        const float2 *hp = hrow ? reinterpret_cast<const float2 *>(hrow + G::kSPL * q) : nullptr;
 #pragma unroll
         for (int k = 0; k < G::kPairs; ++k) {
             const float2 av = __ldg(Ap + k);
             a2[k] = make_float2(av.x * kLog2e, av.y * kLog2e);
-            if (p.h0) h[k] = __ldg(hp + k);
+            if (hp) h[k] = __ldg(hp + k);
         }
     }
 

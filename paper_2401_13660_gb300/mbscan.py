@@ -83,9 +83,10 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
             lib.mb_conv1d_step.argtypes = [vp, vp, vp, vp, vp, i64, i64, ctypes.c_int32, vp]
             lib.mb_scan_backward.argtypes = [ap, vp, vp, vp, ctypes.POINTER(mb_scan_grads), vp, sz, vp]
             lib.mb_selftest_timeout.argtypes = [vp, sz, i64, vp]
+            lib.mb_scan_verify_resume.argtypes = [ap, vp, vp, i64, vp, vp, sz, vp]
             for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_check",
                       "mb_accept_topk", "mb_step_resume", "mb_scan_prefill_ckpt", "mb_scan_backward",
-                      "mb_rmsnorm", "mb_conv1d_step", "mb_selftest_timeout"):
+                      "mb_rmsnorm", "mb_conv1d_step", "mb_selftest_timeout", "mb_scan_verify_resume"):
                 getattr(lib, f).restype = ctypes.c_int
             lib.mb_status_string.argtypes = [ctypes.c_int]
             lib.mb_status_string.restype = ctypes.c_char_p
@@ -235,6 +236,28 @@ def mb_scan_verify(x, dt, B, C, A, y, h_all, *, z=None, D=None, dt_bias=None, h0
     rc = load_library().mb_scan_verify(ctypes.byref(a), _ptr(h_all), _ptr(ws), ws.numel(),
                                        _stream(stream))
     _check(rc, "mb_scan_verify")
+    return y, h_all
+
+
+def mb_scan_verify_resume(x, dt, B, C, A, y, h_all, h_all_prev, accept, *, z=None, D=None, dt_bias=None,
+                          h0=None, ws=None, stream=None, dt_low=None, W_dt=None):
+    """Verify of k = x.shape[1] drafted bytes, stream s starting from h0[s]
+    (zeros if None) when accept[s] == 0, else from h_all_prev[s, accept[s]-1]
+    (the previous verify's per-position states, [batch, k_prev, d_inner,
+    d_state]). A bad accept count is recorded in ws (mb_check) and that stream
+    is left untouched."""
+    a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, h0=h0, dt_low=dt_low, W_dt=W_dt)
+    _need(h_all, "h_all", torch.float32, (a.batch, a.seqlen, a.d_inner, a.d_state), x.device)
+    _need(h_all_prev, "h_all_prev", torch.float32, None, x.device)
+    if h_all_prev.dim() != 4 or h_all_prev.shape[0] != a.batch or \
+            tuple(h_all_prev.shape[2:]) != (a.d_inner, a.d_state):
+        raise ValueError(f"h_all_prev: shape {tuple(h_all_prev.shape)}, expected [batch, k_prev, d_inner, d_state]")
+    _need(accept, "accept", torch.int32, (a.batch,), x.device)
+    if ws is None:
+        ws = new_workspace(a, x.device)
+    rc = load_library().mb_scan_verify_resume(ctypes.byref(a), _ptr(h_all_prev), _ptr(accept), h_all_prev.shape[1],
+                                              _ptr(h_all), _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "mb_scan_verify_resume")
     return y, h_all
 
 

@@ -297,3 +297,22 @@ def test_selftest_timeout_checks():
     assert lib.mb_selftest_timeout(ws + 16, 256, 1000, None) == mb.MB_ERR_INVALID_ARG   # not 256-aligned
     assert lib.mb_selftest_timeout(ws, 256, 0, None) == mb.MB_ERR_INVALID_ARG
     assert lib.mb_selftest_timeout(ws, 256, 5 * 10**9, None) == mb.MB_ERR_INVALID_ARG  # above the kernels' limit
+
+
+def test_verify_resume_checks():
+    lib = mb.load_library()
+    a = _args(L=8)
+    prev, acc, out, ws = FAKE + (30 << 32), FAKE + (31 << 32), FAKE + (32 << 32), FAKE + (200 << 32)
+    call = lambda args=a, p=prev, c=acc, k=4, o=out, w=ws: lib.mb_scan_verify_resume(
+        ctypes.byref(args), p, c, k, o, w, 256, None)
+    assert call() in (mb.MB_OK, mb.MB_ERR_CUDA)               # valid (no GPU here)
+    assert call(w=None) == mb.MB_ERR_INVALID_ARG              # the workspace receives bad counts
+    assert call(k=0) == mb.MB_ERR_INVALID_ARG
+    assert call(p=None) == mb.MB_ERR_INVALID_ARG
+    assert call(c=acc + 2) == mb.MB_ERR_INVALID_ARG           # misaligned accept
+    assert call(o=prev) == mb.MB_ERR_INVALID_ARG              # h_all overlaps h_all_prev
+    assert call(o=a.x) == mb.MB_ERR_INVALID_ARG               # h_all overlaps an input
+    b = _args(L=8)
+    b.y = prev                                                # y overlaps h_all_prev
+    assert call(args=b) == mb.MB_ERR_INVALID_ARG
+    assert call(args=_args(batch=0, L=8)) == mb.MB_OK

@@ -104,3 +104,51 @@ def test_resume_bad_accept_is_reported_and_row_untouched():
                      span["h0"])
     assert rel_err(state[good], rh[good]) <= TOL["bf16"]
     assert rel_err(y[good, 0], ry[good]) <= TOL["bf16"]
+
+
+# ------------------------------------------------------------------ verify resume
+def _next_span(batch, k2, Dn, dtype, seed):
+    return make_inputs(batch, k2, Dn, 16, dtype, "zeros", seed=seed, device=DEV)
+
+
+@pytest.mark.parametrize("dtype, batch, k, k2, Dn, with_h0", [("bf16", 32, 16, 16, 2048, True),
+                                                              ("f32", 7, 5, 19, 72, True),
+                                                              ("bf16", 5, 3, 8, 8 * 67, False)])
+def test_verify_resume_equals_rollback_then_verify(dtype, batch, k, k2, Dn, with_h0):
+    """mb_scan_verify_resume is bit for bit mb_rollback then mb_scan_verify
+    (the same scan from the same starting states), and matches the oracle."""
+    span, _, h_all, acc = _problem(batch, k, Dn, dtype, h0="normal" if with_h0 else "zeros", seed=60 + k)
+    h0 = span["h0"] if with_h0 else None
+    nxt = _next_span(batch, k2, Dn, dtype, seed=70 + k2)
+    y = torch.empty_like(nxt["x"])
+    h_all2 = torch.empty(batch, k2, Dn, 16, device=DEV)
+    mb.mb_scan_verify_resume(nxt["x"], nxt["dt"], nxt["B"], nxt["C"], span["A"], y, h_all2, h_all, acc,
+                             z=nxt["z"], D=span["D"], dt_bias=span["dt_bias"], h0=h0)
+    kept = torch.empty(batch, Dn, 16, device=DEV)
+    mb.mb_rollback(h0 if h0 is not None else torch.zeros_like(kept), h_all, acc, kept)
+    y_ref = torch.empty_like(nxt["x"])
+    h_ref = torch.empty_like(h_all2)
+    mb.mb_scan_verify(nxt["x"], nxt["dt"], nxt["B"], nxt["C"], span["A"], y_ref, h_ref, z=nxt["z"],
+                      D=span["D"], dt_bias=span["dt_bias"], h0=kept)
+    assert torch.equal(y, y_ref) and torch.equal(h_all2, h_ref)
+    start = oracle.rollback(to_np(h0) if h0 is not None else np.zeros((batch, Dn, 16)), to_np(h_all),
+                            acc.cpu().numpy())
+    ry, _, rall = oracle.scan(to_np(nxt["x"]), to_np(nxt["dt"]), to_np(nxt["B"]), to_np(nxt["C"]),
+                              to_np(span["A"]), z=to_np(nxt["z"]), D=to_np(span["D"]),
+                              dt_bias=to_np(span["dt_bias"]), h0=start, want_h_all=True)
+    assert rel_err(y, ry) <= TOL[dtype] and rel_err(h_all2, rall) <= TOL[dtype]
+
+
+def test_verify_resume_bad_accept_is_reported_and_stream_untouched():
+    span, _, h_all, acc = _problem(4, 6, 96, "f32", seed=81)
+    nxt = _next_span(4, 8, 96, "f32", seed=82)
+    acc[2] = 7                                    # > k_prev = 6
+    y = torch.full_like(nxt["x"], 5.0)
+    h_all2 = torch.full((4, 8, 96, 16), 5.0, device=DEV)
+    ws = torch.zeros(256, dtype=torch.uint8, device=DEV)
+    mb.mb_scan_verify_resume(nxt["x"], nxt["dt"], nxt["B"], nxt["C"], span["A"], y, h_all2, h_all, acc,
+                             z=nxt["z"], D=span["D"], dt_bias=span["dt_bias"], h0=span["h0"], ws=ws)
+    assert mb.mb_check(ws) == (mb.MB_ERR_INVALID_ARG, 2)
+    assert torch.equal(y[2], torch.full_like(y[2], 5.0))
+    assert torch.equal(h_all2[2], torch.full_like(h_all2[2], 5.0))
+    assert not torch.equal(y[1], torch.full_like(y[1], 5.0))   # the other streams were scanned
