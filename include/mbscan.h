@@ -104,11 +104,16 @@ typedef struct {
     int32_t dt_low_stride;
 } mb_scan_args;
 
-/* Bytes of device workspace that mb_scan_prefill / mb_scan_verify need for
- * `args` (a status block written by bounded device-side waits). The caller
- * allocates it (256-byte aligned) and may reuse it across calls on one
- * stream; calls that overlap on the GPU need distinct workspaces. Returns 0
- * for invalid arguments. */
+/* Bytes of device workspace to pass with `args`: a 256-byte status block
+ * (written by bounded device-side waits), plus, when the batch rows and
+ * channels of a long span fill less than half of the GPU, scratch that lets
+ * mb_scan_prefill split the span over L (two passes: per-segment summaries,
+ * then the scan of every segment from its folded start state; Section 2's
+ * associative operator). Any workspace of at least 256 bytes is accepted: a
+ * smaller one than this runs such spans unsplit. The caller allocates it
+ * (256-byte aligned) and may reuse it across calls on one stream; calls that
+ * overlap on the GPU need distinct workspaces. Returns 0 for invalid
+ * arguments. */
 size_t mb_workspace_size(const mb_scan_args *args);
 
 /*
@@ -117,9 +122,10 @@ size_t mb_workspace_size(const mb_scan_args *args);
  * channel, writes y and, if h_last != NULL, the final state
  * h_last[batch, d_inner, d_state] fp32 (the state MambaByte caches to resume
  * generation). h_last may alias h0.
- *   ws, ws_bytes : workspace of at least mb_workspace_size(args) bytes; it
- *                  must start zeroed once after allocation and is left zeroed
- *                  by every successful call.
+ *   ws, ws_bytes : workspace of at least 256 bytes (mb_workspace_size(args)
+ *                  for the split of long few-channel spans); its status block
+ *                  (first 256 bytes) must start zeroed once after allocation
+ *                  and is left zeroed by every successful call.
  */
 mb_status mb_scan_prefill(const mb_scan_args *args, float *h_last, void *ws, size_t ws_bytes,
                           void *stream);

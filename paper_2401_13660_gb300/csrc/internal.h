@@ -37,6 +37,11 @@ struct ScanParams {
     const float *h_prev_all;
     const int32_t *accept;
     int64_t k_prev;
+    // Time split of a prefill over nseg segments of L (1: not split): seg_h,
+    // seg_p [batch, nseg, d_inner, 16] hold each segment's end state from a
+    // zero start and the product of its decays (scratch in the workspace).
+    int64_t nseg;
+    float *seg_h, *seg_p;
 };
 
 constexpr int kRankTile = 64;    // dt_rank elements per 128-byte swizzled TMA box
@@ -61,6 +66,11 @@ constexpr long long kMaxWaitCycles = 4000000000LL;   // the kernels' wait limit 
 // Bounded-wait diagnostic (selftest.cu): a wait that runs out after `limit` clocks.
 cudaError_t launch_wait_timeout(StatusBlock *sb, long long limit, cudaStream_t s);
 cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s);
+// Segments a prefill of these sizes is split into when the workspace has room
+// (1 when the batch rows and channels alone fill the GPU), and the scratch
+// bytes that split needs beyond the status block.
+int64_t prefill_segments(const ScanParams &p, bool bf16);
+size_t prefill_split_bytes(const ScanParams &p, int64_t nseg);
 cudaError_t launch_verify(const ScanParams &p, bool bf16, cudaStream_t s);
 // Prefill that also writes p.h_ckpt [batch, ceil(L / kCkptSteps), d_inner, 16].
 cudaError_t launch_prefill_ckpt(const ScanParams &p, bool bf16, cudaStream_t s);

@@ -123,13 +123,16 @@ ScanParams to_params(const mb_scan_args *a, float *h_out, StatusBlock *status) {
     p.h_prev_all = nullptr;
     p.accept = nullptr;
     p.k_prev = 0;
+    p.nseg = 1;
+    p.seg_h = p.seg_p = nullptr;
     return p;
 }
 
+// The status block must fit; a larger workspace (mb_workspace_size) only
+// lets mb_scan_prefill split long few-channel spans.
 mb_status check_ws(const mb_scan_args *a, void *ws, size_t ws_bytes) {
-    const size_t need = mb_workspace_size(a);
-    if (need == 0) return MB_OK;
-    if (ws == nullptr || ws_bytes < need) return MB_ERR_INVALID_ARG;
+    if (mb_workspace_size(a) == 0) return MB_OK;
+    if (ws == nullptr || ws_bytes < mbscan::kStatusBytes) return MB_ERR_INVALID_ARG;
     if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return MB_ERR_INVALID_ARG;
     return MB_OK;
 }
@@ -142,7 +145,9 @@ extern "C" {
 
 size_t mb_workspace_size(const mb_scan_args *args) {
     if (check_args(args, false, false) != MB_OK) return 0;
-    return mbscan::kStatusBytes;
+    const ScanParams p = to_params(args, nullptr, nullptr);
+    const bool bf16 = args->dtype == MB_BF16;
+    return mbscan::kStatusBytes + mbscan::prefill_split_bytes(p, mbscan::prefill_segments(p, bf16));
 }
 
 mb_status mb_scan_prefill(const mb_scan_args *args, float *h_last, void *ws, size_t ws_bytes,
@@ -166,7 +171,28 @@ mb_status mb_scan_prefill(const mb_scan_args *args, float *h_last, void *ws, siz
     }
     if (args->batch * args->d_inner == 0) return MB_OK;
     ScanParams p = to_params(args, h_last, static_cast<StatusBlock *>(ws));
-    return from_cuda(mbscan::launch_prefill(p, args->dtype == MB_BF16, (cudaStream_t)stream));
+    const bool bf16 = args->dtype == MB_BF16;
+    // Long spans with few channels are split over L when the workspace holds
+    // the segment summaries (after the status block); else they run unsplit.
+    const int64_t nseg = mbscan::prefill_segments(p, bf16);
+    const size_t split = mbscan::prefill_split_bytes(p, nseg);
+    if (nseg > 1 && ws_bytes >= mbscan::kStatusBytes + split) {
+        const int64_t es = bf16 ? 2 : 4;
+        const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
+        const int64_t sbytes = args->batch * args->d_inner * args->d_state * 4;
+        const Range rs = range_of(static_cast<char *>(ws) + mbscan::kStatusBytes, (int64_t)split);
+        const Range others[] = {range_of(args->x, tok), range_of(args->z, tok), range_of(args->dt, tok),
+                                range_of(args->y, tok), range_of(args->B, bc_bytes(args)),
+                                range_of(args->C, bc_bytes(args)), range_of(args->h0, sbytes),
+                                range_of(h_last, sbytes), range_of(args->A, args->d_inner * args->d_state * 4),
+                                range_of(args->D, args->d_inner * 4), range_of(args->dt_bias, args->d_inner * 4)};
+        for (const Range &r : others)
+            if (overlap(rs, r)) return MB_ERR_INVALID_ARG;
+        p.nseg = nseg;
+        p.seg_h = reinterpret_cast<float *>(static_cast<char *>(ws) + mbscan::kStatusBytes);
+        p.seg_p = p.seg_h + split / (2 * sizeof(float));
+    }
+    return from_cuda(mbscan::launch_prefill(p, bf16, (cudaStream_t)stream));
 }
 
 mb_status mb_scan_verify(const mb_scan_args *args, float *h_all, void *ws, size_t ws_bytes,

@@ -113,6 +113,7 @@ struct PrefillArgs {
     ScanParams p;
     int has_gate;
     int nbox;      // ceil(dt_rank / kRankTile)
+    int grid_segs; // segments of L covered by the grid (blockIdx = (b, segment, channel tile))
 };
 
 // Shared-memory layout of the fused Delta projection, after the Smem struct:
@@ -265,7 +266,12 @@ __device__ __forceinline__ float reduce_steps(const float (&part)[LPC], int q) {
     }
 }
 
-template <typename T, int LPC, int STAGES, bool kStoreAll, bool kCkpt, bool kFuse>
+// kSummary (first pass of a time-split prefill): scan each segment of L from a
+// zero state and record its end state and the product of its decays in the
+// scratch (no outputs). The second pass is the plain kernel: its segment s
+// starts from the state the summaries of segments 0 .. s-1 give (folded with
+// the associative operator of Section 2: h <- P_s' * h + H_s').
+template <typename T, int LPC, int STAGES, bool kStoreAll, bool kCkpt, bool kFuse, bool kSummary = false>
 __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED_MINB : MB_VERIFY_MINB) : 1)
     prefill_kernel(const __grid_constant__ PrefillArgs a) {
     using G = Geom<LPC>;
@@ -290,12 +296,23 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
     const ScanParams &p = a.p;
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
-    // blockIdx.x = batch row * channel tiles + channel tile (no 65535 limit on batch)
+    // blockIdx.x = (batch row, segment of L, channel tile), channel tile fastest;
+    // only the plain prefill is ever split over L
+    constexpr bool kSplit = !kStoreAll && !kCkpt && !kFuse;
     const int ntd = (int)((p.d_inner + CH - 1) / CH);
-    const int b = blockIdx.x / ntd;
-    const int d0 = (blockIdx.x % ntd) * CH;
     const int64_t L = p.seqlen, D = p.d_inner;
-    const int64_t nchunks = (L + kT - 1) / kT;
+    const int64_t nchunks = (L + kT - 1) / kT;   // chunks of the whole span
+    int seg = 0, b = (int)(blockIdx.x / ntd);
+    int64_t nseg = 1, c0 = 0, nch = nchunks;    // this CTA's chunks: c0 .. c0 + nch - 1
+    if constexpr (kSplit) {
+        seg = (int)((blockIdx.x / ntd) % a.grid_segs);
+        b = (int)(blockIdx.x / ntd / a.grid_segs);
+        nseg = p.nseg > 1 ? p.nseg : 1;
+        const int64_t cps = (nchunks + nseg - 1) / nseg;   // chunks per segment
+        c0 = seg * cps;
+        nch = nchunks - c0 < cps ? nchunks - c0 : cps;
+    }
+    const int d0 = (blockIdx.x % ntd) * CH;
     const bool gate = a.has_gate != 0;
 
     if (tid == 0) {
@@ -316,11 +333,11 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
         }
     }
     if (tid == 0) {
-        for (int st = 0; st < STAGES && st < nchunks; ++st) {
+        for (int st = 0; st < STAGES && st < nch; ++st) {
             // the CTA's W_dt slice rides on chunk 0's barrier (its bytes are
             // part of that arrival's expected count)
             const bool wslice = kFuse && st == 0;
-            issue_chunk(s, a, st, st, d0, b, fz, wslice ? (uint32_t)a.nbox * FuseLayout<CH>::kWBox : 0u);
+            issue_chunk(s, a, st, c0 + st, d0, b, fz, wslice ? (uint32_t)a.nbox * FuseLayout<CH>::kWBox : 0u);
             if (wslice)
                 for (int bx = 0; bx < a.nbox; ++bx)
                     tma_load_2d(fz + (uint32_t)(STAGES * a.nbox) * kDtlBox + (uint32_t)bx * FuseLayout<CH>::kWBox,
@@ -363,30 +380,42 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
         for (int k = 0; k < G::kPairs; ++k) {
             const float2 av = __ldg(Ap + k);
             a2[k] = make_float2(av.x * kLog2e, av.y * kLog2e);
-            if (hp) h[k] = __ldg(hp + k);
+            if (hp && !kSummary) h[k] = __ldg(hp + k);   // a summary starts from zero
+        }
+        if constexpr (kSplit && !kSummary) {   // segment s > 0 of a split span: fold the summaries before it
+            for (int sp = 0; sp < seg; ++sp) {
+                const int64_t off = (((int64_t)b * nseg + sp) * D + d) * kDState + G::kSPL * q;
+                const float2 *hs_ = reinterpret_cast<const float2 *>(p.seg_h + off);
+                const float2 *ps_ = reinterpret_cast<const float2 *>(p.seg_p + off);
+#pragma unroll
+                for (int k = 0; k < G::kPairs; ++k) h[k] = fma2(ps_[k], h[k], hs_[k]);
+            }
         }
     }
+    float2 prod[G::kPairs];   // kSummary: product of the segment's decays
+#pragma unroll
+    for (int k = 0; k < G::kPairs; ++k) prod[k] = make_float2(1.f, 1.f);
 
     // ---- prologue: chunk 0
-    bool ok = nchunks > 0 ? mbar_wait(&s.full[0], 0) : true;
+    bool ok = nch > 0 ? mbar_wait(&s.full[0], 0) : true;
     if constexpr (kFuse) ok = __all_sync(kFull, ok);   // mma.sync needs the whole warp
     auto stage_fx = [&](int st) {   // the fused projection's operands for ring stage st
         FuseCtx f = fx;
         if constexpr (kFuse) f.dtl = fz_addr + (uint32_t)(st * a.nbox) * kDtlBox;
         return f;
     };
-    if (ok && nchunks > 0) convert(s.cv[0], s.raw[0], cr, 0, L, gate, stage_fx(0));
+    if (ok && nch > 0) convert(s.cv[0], s.raw[0], cr, c0 * kT, L, gate, stage_fx(0));
     if (__syncthreads_or(ok ? 0 : 1)) {
         if (tid == 0) {
             report(p.status, 4 /* MB_ERR_TIMEOUT */, 0);
-            for (int j = 0; j < STAGES && j < nchunks; ++j) mbar_wait(&s.full[j], 0);
+            for (int j = 0; j < STAGES && j < nch; ++j) mbar_wait(&s.full[j], 0);
         }
         return;
     }
 
-    for (int64_t i = 0; i < nchunks; ++i) {
-        const int64_t t0 = i * kT;
-        const bool has_next = i + 1 < nchunks;
+    for (int64_t i = 0; i < nch; ++i) {   // i: chunk c0 + i of the span, ring slot i % STAGES
+        const int64_t t0 = (c0 + i) * kT;
+        const bool has_next = i + 1 < nch;
         // (1) chunk i+1: wait for its tiles and convert them
         const int nst = (int)((i + 1) % STAGES);
         ok = has_next ? mbar_wait(&s.full[nst], (uint32_t)(((i + 1) / STAGES) & 1)) : true;
@@ -398,7 +427,7 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
             static_assert(kT == kCkptSteps, "checkpoints are taken per chunk");
             if (chan_ok) {
                 float2 *dst = reinterpret_cast<float2 *>(
-                    p.h_ckpt + (((int64_t)b * nchunks + i) * D + d) * kDState + G::kSPL * q);
+                    p.h_ckpt + (((int64_t)b * nchunks + c0 + i) * D + d) * kDState + G::kSPL * q);
 #pragma unroll
                 for (int k = 0; k < G::kPairs; k += 2)
                     *reinterpret_cast<float4 *>(dst + k) = make_float4(h[k].x, h[k].y, h[k + 1].x, h[k + 1].y);
@@ -435,10 +464,13 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
 #pragma unroll
             for (int k = 0; k < G::kPairs; ++k) {
                 h[k] = fma2(ab[t][k], h[k], mul2(bp[k], gg));
-                acc[k & 1] = k < 2 ? mul2(cp[k], h[k]) : fma2(cp[k], h[k], acc[k & 1]);
+                if constexpr (kSummary) prod[k] = mul2(prod[k], ab[t][k]);
+                else acc[k & 1] = k < 2 ? mul2(cp[k], h[k]) : fma2(cp[k], h[k], acc[k & 1]);
             }
-            const float2 sum = add2(acc[0], acc[1]);
-            part[t] = sum.x + sum.y;
+            if constexpr (!kSummary) {
+                const float2 sum = add2(acc[0], acc[1]);
+                part[t] = sum.x + sum.y;
+            }
             if constexpr (kStoreAll) {
                 if (chan_ok && t0 + t < L) {
                     float2 *dst = reinterpret_cast<float2 *>(
@@ -453,7 +485,7 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
         // (3) chunk i: reduce across the lanes of each channel, gate, stage y
         T(&ys)[kT][CH] = s.ys[i & 1];
 #pragma unroll
-        for (int m = 0; m < kT / LPC; ++m) {
+        for (int m = 0; m < (kSummary ? 0 : kT / LPC); ++m) {
             float grp[LPC];
 #pragma unroll
             for (int u = 0; u < LPC; ++u) grp[u] = part[LPC * m + u];
@@ -466,27 +498,37 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
         if (tid == 0) bulk_wait_read_all();   // the store of chunk i-1 no longer reads its tile
         if (__syncthreads_or(ok ? 0 : 1)) {
             if (tid == 0) {
-                report(p.status, 4 /* MB_ERR_TIMEOUT */, i + 1);
-                for (int64_t j = i + 1; j < i + STAGES && j < nchunks; ++j)
+                report(p.status, 4 /* MB_ERR_TIMEOUT */, c0 + i + 1);
+                for (int64_t j = i + 1; j < i + STAGES && j < nch; ++j)
                     mbar_wait(&s.full[j % STAGES], (uint32_t)((j / STAGES) & 1));
                 bulk_wait_all();
             }
             return;
         }
         if (tid == 0) {
-            tma_store_3d(&a.tm_y, &ys[0][0], d0, (int)t0, b);
-            bulk_commit();
+            if constexpr (!kSummary) {
+                tma_store_3d(&a.tm_y, &ys[0][0], d0, (int)t0, b);
+                bulk_commit();
+            }
             // stage i % STAGES (chunk i: converted last iteration, scanned
             // now) is free: refill it with chunk i + STAGES
-            if (i + STAGES < nchunks) {
+            if (i + STAGES < nch) {
                 fence_proxy_async_smem();
-                issue_chunk(s, a, (int)(i % STAGES), i + STAGES, d0, b, fz);
+                issue_chunk(s, a, (int)(i % STAGES), c0 + i + STAGES, d0, b, fz);
             }
         }
     }
     if (tid == 0) bulk_wait_all();
 
-    if (!kStoreAll && p.h_out && chan_ok) {
+    if constexpr (kSummary) {   // this segment's end state from a zero start, and its decay product
+        if (chan_ok) {
+            const int64_t off = (((int64_t)b * nseg + seg) * D + d) * kDState + G::kSPL * q;
+            float2 *hd = reinterpret_cast<float2 *>(p.seg_h + off);
+            float2 *pd = reinterpret_cast<float2 *>(p.seg_p + off);
+#pragma unroll
+            for (int k = 0; k < G::kPairs; ++k) { hd[k] = h[k]; pd[k] = prod[k]; }
+        }
+    } else if (!kStoreAll && p.h_out && chan_ok && seg == nseg - 1) {   // the span's last state
         float2 *hp = reinterpret_cast<float2 *>(p.h_out + ((int64_t)b * D + d) * kDState + G::kSPL * q);
 #pragma unroll
         for (int k = 0; k < G::kPairs; ++k) hp[k] = h[k];
@@ -516,6 +558,9 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
     memset(&a, 0, sizeof(a));
     a.p = p;
     a.has_gate = p.z != nullptr;
+    constexpr bool kSplittable = !kStoreAll && !kCkpt && !kFuse;
+    if (!kSplittable || p.nseg < 2 || !p.seg_h || !p.seg_p) a.p.nseg = 1;
+    const int64_t nseg = a.p.nseg;
     size_t fuse_bytes = 0;
     if constexpr (kFuse) {
         // dt_low [batch, L, r] (rows dt_low_stride apart) and W_dt [D, r], both
@@ -541,14 +586,65 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
         !make_map(&a.tm_y, p.y, bf16, p.batch, p.seqlen, p.d_inner, kCh))
         return cudaErrorInvalidValue;
     const size_t smem = sizeof(Smem<T, kCh, STAGES, kFuse>) + 128 + fuse_bytes;
+    const int64_t ctas = ((p.d_inner + kCh - 1) / kCh) * p.batch;   // per segment of L
+    cudaError_t e;
+    if constexpr (kSplittable) {
+        if (nseg > 1) {   // first pass: summaries of segments 0 .. nseg-2
+            PrefillArgs a1 = a;
+            a1.has_gate = 0;   // no outputs: the gate is not read
+            a1.grid_segs = (int)(nseg - 1);
+            auto k1 = prefill_kernel<T, LPC, STAGES, false, false, false, true>;
+            if ((e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+                return e;
+            if ((e = launch_pdl(false, k1, dim3((unsigned)(ctas * (nseg - 1))), dim3(kThreads), smem, s, a1)) !=
+                cudaSuccess)
+                return e;
+        }
+    }
+    a.grid_segs = (int)nseg;
     auto k = prefill_kernel<T, LPC, STAGES, kStoreAll, kCkpt, kFuse>;
-    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    const dim3 grid((unsigned)(((p.d_inner + kCh - 1) / kCh) * p.batch));
-    return launch_pdl(false, k, grid, dim3(kThreads), smem, s, a);
+    return launch_pdl(false, k, dim3((unsigned)(ctas * nseg)), dim3(kThreads), smem, s, a);
 }
 
 }  // namespace
+
+// Time split: only when the batch rows and channel tiles give at most one CTA
+// per SM (a CTA alone on an SM runs a chunk in ~1.1 us, four together take
+// ~2 us each: the SM idles); then into as many segments as fill the resident
+// slots (4 per SM for bf16 at 118 registers, 3 for fp32), each at least
+// kMinSegChunks chunks long. The summary pass costs ~70 % of a scan, so at 1.7
+// CTAs per SM (batch 4 x 2048 channels) the split measured slower (677 -> 766 us)
+// while batch 1 x 2048 channels x 8192 steps went 554 -> 212 us.
+constexpr int64_t kMinSegChunks = 8;
+
+int64_t prefill_segments(const ScanParams &p, bool bf16) {
+    if (p.batch <= 0 || p.d_inner <= 0 || p.seqlen <= 0 || p.dt_low) return 1;
+    constexpr int kMaxDevices = 64;
+    static int sm_count[kMaxDevices] = {0};   // per device, filled on first use
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 1;
+    if (sm_count[dev] == 0) {
+        int v = 0;
+        if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) return 1;
+        sm_count[dev] = v;
+    }
+    constexpr int kCh = Geom<kPrefillLanesPerChannel>::kCh;
+    const int64_t slots = (int64_t)sm_count[dev] * (bf16 ? 4 : 3);
+    const int64_t ctas = p.batch * ((p.d_inner + kCh - 1) / kCh);
+    if (ctas > sm_count[dev]) return 1;
+    const int64_t nchunks = (p.seqlen + kT - 1) / kT;
+    int64_t nseg = slots / ctas;
+    if (nseg > nchunks / kMinSegChunks) nseg = nchunks / kMinSegChunks;
+    if (nseg < 2) return 1;
+    const int64_t cps = (nchunks + nseg - 1) / nseg;
+    return (nchunks + cps - 1) / cps;   // no empty segment
+}
+
+size_t prefill_split_bytes(const ScanParams &p, int64_t nseg) {
+    return nseg > 1 ? (size_t)(2 * p.batch * nseg * p.d_inner * kDState) * sizeof(float) : 0;
+}
 
 cudaError_t launch_prefill(const ScanParams &p, bool bf16, cudaStream_t s) {
     if (p.batch == 0 || p.d_inner == 0) return cudaSuccess;
