@@ -137,6 +137,30 @@ mb_status check_ws(const mb_scan_args *a, void *ws, size_t ws_bytes) {
     return MB_OK;
 }
 
+// Long spans with few channels are split over L when the workspace holds the
+// segment summaries (after the status block); else they run unsplit.
+mb_status setup_split(const mb_scan_args *args, ScanParams &p, const float *h_last, void *ws, size_t ws_bytes) {
+    const bool bf16 = args->dtype == MB_BF16;
+    const int64_t nseg = mbscan::prefill_segments(p, bf16);
+    const size_t split = mbscan::prefill_split_bytes(p, nseg);
+    if (nseg < 2 || ws_bytes < mbscan::kStatusBytes + split) return MB_OK;
+    const int64_t es = bf16 ? 2 : 4;
+    const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
+    const int64_t sbytes = args->batch * args->d_inner * args->d_state * 4;
+    const Range rs = range_of(static_cast<char *>(ws) + mbscan::kStatusBytes, (int64_t)split);
+    const Range others[] = {range_of(args->x, tok), range_of(args->z, tok), range_of(args->dt, tok),
+                            range_of(args->y, tok), range_of(args->B, bc_bytes(args)),
+                            range_of(args->C, bc_bytes(args)), range_of(args->h0, sbytes), range_of(h_last, sbytes),
+                            range_of(args->A, args->d_inner * args->d_state * 4),
+                            range_of(args->D, args->d_inner * 4), range_of(args->dt_bias, args->d_inner * 4)};
+    for (const Range &r : others)
+        if (overlap(rs, r)) return MB_ERR_INVALID_ARG;
+    p.nseg = nseg;
+    p.seg_h = reinterpret_cast<float *>(static_cast<char *>(ws) + mbscan::kStatusBytes);
+    p.seg_p = p.seg_h + split / (2 * sizeof(float));
+    return MB_OK;
+}
+
 mb_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MB_OK : MB_ERR_CUDA; }
 
 }  // namespace
@@ -172,26 +196,7 @@ mb_status mb_scan_prefill(const mb_scan_args *args, float *h_last, void *ws, siz
     if (args->batch * args->d_inner == 0) return MB_OK;
     ScanParams p = to_params(args, h_last, static_cast<StatusBlock *>(ws));
     const bool bf16 = args->dtype == MB_BF16;
-    // Long spans with few channels are split over L when the workspace holds
-    // the segment summaries (after the status block); else they run unsplit.
-    const int64_t nseg = mbscan::prefill_segments(p, bf16);
-    const size_t split = mbscan::prefill_split_bytes(p, nseg);
-    if (nseg > 1 && ws_bytes >= mbscan::kStatusBytes + split) {
-        const int64_t es = bf16 ? 2 : 4;
-        const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
-        const int64_t sbytes = args->batch * args->d_inner * args->d_state * 4;
-        const Range rs = range_of(static_cast<char *>(ws) + mbscan::kStatusBytes, (int64_t)split);
-        const Range others[] = {range_of(args->x, tok), range_of(args->z, tok), range_of(args->dt, tok),
-                                range_of(args->y, tok), range_of(args->B, bc_bytes(args)),
-                                range_of(args->C, bc_bytes(args)), range_of(args->h0, sbytes),
-                                range_of(h_last, sbytes), range_of(args->A, args->d_inner * args->d_state * 4),
-                                range_of(args->D, args->d_inner * 4), range_of(args->dt_bias, args->d_inner * 4)};
-        for (const Range &r : others)
-            if (overlap(rs, r)) return MB_ERR_INVALID_ARG;
-        p.nseg = nseg;
-        p.seg_h = reinterpret_cast<float *>(static_cast<char *>(ws) + mbscan::kStatusBytes);
-        p.seg_p = p.seg_h + split / (2 * sizeof(float));
-    }
+    if ((st = setup_split(args, p, h_last, ws, ws_bytes)) != MB_OK) return st;
     return from_cuda(mbscan::launch_prefill(p, bf16, (cudaStream_t)stream));
 }
 
@@ -373,6 +378,9 @@ mb_status mb_scan_prefill_ckpt(const mb_scan_args *args, float *h_last, float *h
         return MB_ERR_INVALID_ARG;
     ScanParams p = to_params(args, h_last, static_cast<StatusBlock *>(ws));
     p.h_ckpt = h_ckpt;
+    if ((st = setup_split(args, p, h_last, ws, ws_bytes)) != MB_OK) return st;
+    if (p.nseg > 1 && overlap(rc, range_of(p.seg_h, (int64_t)mbscan::prefill_split_bytes(p, p.nseg))))
+        return MB_ERR_INVALID_ARG;
     return from_cuda(mbscan::launch_prefill_ckpt(p, args->dtype == MB_BF16, (cudaStream_t)stream));
 }
 

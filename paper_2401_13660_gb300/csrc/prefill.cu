@@ -298,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
     const int warp = tid >> 5, lane = tid & 31;
     // blockIdx.x = (batch row, segment of L, channel tile), channel tile fastest;
     // only the plain prefill is ever split over L
-    constexpr bool kSplit = !kStoreAll && !kCkpt && !kFuse;
+    constexpr bool kSplit = !kStoreAll && !kFuse;
     const int ntd = (int)((p.d_inner + CH - 1) / CH);
     const int64_t L = p.seqlen, D = p.d_inner;
     const int64_t nchunks = (L + kT - 1) / kT;   // chunks of the whole span
@@ -558,7 +558,7 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
     memset(&a, 0, sizeof(a));
     a.p = p;
     a.has_gate = p.z != nullptr;
-    constexpr bool kSplittable = !kStoreAll && !kCkpt && !kFuse;
+    constexpr bool kSplittable = !kStoreAll && !kFuse;
     if (!kSplittable || p.nseg < 2 || !p.seg_h || !p.seg_p) a.p.nseg = 1;
     const int64_t nseg = a.p.nseg;
     size_t fuse_bytes = 0;

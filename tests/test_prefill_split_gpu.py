@@ -67,3 +67,31 @@ def test_wide_spans_are_not_split():
     inp = make_inputs(8, 256, 2048, 16, "bf16", "zeros", seed=98, device=DEV)
     _, n = _ws(inp)
     assert n == 256   # 8 rows x 64 tiles already fill the GPU
+
+
+def test_split_training_forward_checkpoints_and_backward():
+    """The checkpointed forward splits the same way; its checkpoints (the
+    state before every 16-step chunk) and the backward that reads them match
+    the unsplit forward's."""
+    inp = make_inputs(1, 1500, 64, 16, "f32", "normal", seed=99, device=DEV)
+    x = inp["x"]
+    out = {}
+    for split in (True, False):
+        ws, n = _ws(inp, split)
+        assert (n > 256) == split
+        y = torch.empty_like(x)
+        hl = torch.empty(1, 64, 16, device=DEV)
+        _, _, ck = mb.mb_scan_prefill_ckpt(x, inp["dt"], inp["B"], inp["C"], inp["A"], y, z=inp["z"], D=inp["D"],
+                                           dt_bias=inp["dt_bias"], h0=inp["h0"], h_last=hl, ws=ws)
+        g = torch.Generator(device=DEV).manual_seed(5)
+        dout = torch.randn(x.shape, device=DEV, generator=g)
+        grads = mb.mb_scan_backward(x, inp["dt"], inp["B"], inp["C"], inp["A"], ck, dout, z=inp["z"], D=inp["D"],
+                                    dt_bias=inp["dt_bias"], h0=inp["h0"])
+        out[split] = (y, hl, ck, grads)
+    y, hl, ck, gr = out[True]
+    y1, hl1, ck1, gr1 = out[False]
+    torch.testing.assert_close(ck, ck1, rtol=1e-4, atol=1e-5)
+    torch.testing.assert_close(y, y1, rtol=1e-4, atol=1e-4)
+    torch.testing.assert_close(hl, hl1, rtol=1e-4, atol=1e-5)
+    for k in ("dx", "ddt", "dz", "dB", "dC", "dA", "dh0"):
+        assert rel_err(gr[k], gr1[k].double().cpu().numpy()) <= 1e-3, k
