@@ -200,6 +200,13 @@ mb_status mb_accept_topk(const void *logits, int32_t dtype, const uint8_t *draft
  * `state` [batch, d_inner, d_state] fp32 is read and updated in place; y is
  * [batch, 1, d_inner]. Used for the corrector loop of Algorithm 1 and for
  * plain generation.
+ * Launch overlap: the step kernel is launched with programmatic dependent
+ * launch. It waits for the previous kernel on the stream to complete before
+ * touching memory, and lets the next kernel launch while it runs. A kernel
+ * the caller launches next with programmatic stream serialization must
+ * therefore execute griddepcontrol.wait (cudaGridDependencySynchronize)
+ * before reading y or state, as CUDA requires for any such launch. Plainly
+ * launched work is ordered as usual.
  */
 mb_status mb_step(const mb_scan_args *args, float *state, void *stream);
 
