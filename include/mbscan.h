@@ -224,10 +224,11 @@ mb_status mb_step(const mb_scan_args *args, float *state, void *stream);
  *   accept  : [batch] int32 device array, values in [0, k] (mb_accept_topk)
  *   state   : [batch, d_inner, d_state] fp32 output; may alias args->h0, not
  *             h_all
- *   ws      : workspace (mb_workspace_size(args) bytes, 256-byte aligned) or
- *             NULL; an accept count outside [0, k] is a caller error: that
- *             stream's state and y are left untouched and the first such
- *             stream index is recorded in ws's status block (mb_check).
+ *   ws      : workspace (at least 256 bytes, 256-byte aligned) or NULL; an
+ *             accept count outside [0, k] is a caller error: that stream's
+ *             state and y are left untouched and the first such stream index
+ *             is recorded in ws's status block (mb_check).
+ * Launched with the same launch overlap as mb_step.
  */
 mb_status mb_step_resume(const mb_scan_args *args, const float *h_all, const int32_t *accept,
                          int64_t k, float *state, void *ws, size_t ws_bytes, void *stream);
