@@ -202,8 +202,7 @@ template <typename T>
 __global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_constant__ BwdArgs a) {
     constexpr int S = kBStages;
     extern __shared__ unsigned char smem_dyn[];
-    BSmem<T> &s = *reinterpret_cast<BSmem<T> *>((reinterpret_cast<uintptr_t>(smem_dyn) + 127) &
-                                                ~static_cast<uintptr_t>(127));
+    BSmem<T> &s = smem_aligned<BSmem<T>>(smem_dyn);
     const ScanParams &p = a.p;
     const GradParams &gp = a.g;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;

@@ -105,8 +105,7 @@ __device__ __forceinline__ float4 lds4(const __nv_bfloat16 *p) {
 template <typename T, bool kResume>
 __global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constant__ StepArgs a) {
     extern __shared__ unsigned char smem_dyn[];
-    StepSmem<T> &s = *reinterpret_cast<StepSmem<T> *>(
-        (reinterpret_cast<uintptr_t>(smem_dyn) + 127) & ~static_cast<uintptr_t>(127));
+    StepSmem<T> &s = smem_aligned<StepSmem<T>>(smem_dyn);
     const ScanParams &p = a.p;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t D = p.d_inner;

@@ -23,11 +23,13 @@
 //    waits, tma.cuh);
 //  * the CTA converts a chunk once per (t, channel) into fp32 in shared
 //    memory: (Delta, Delta*x) with Delta = softplus(dt + bias), (D*x, silu z);
+//    a bf16 prefill also widens the chunk's B and C rows to fp32 once, so
+//    that the scan does not convert them again in every lane;
 //  * each lane scans the chunk: Abar = 2^(Delta * A*log2 e) on the SFU for all
 //    kT steps, then h = Abar*h + B*(Delta*x) and its share of C.h in packed
-//    f32x2 arithmetic, reading B and C straight from the TMA tile in the input
-//    dtype (for bf16 this halves the shared-memory bytes of the scan, whose
-//    bandwidth is its limit); groups of LPC steps are reduced across the LPC
+//    f32x2 arithmetic, reading B and C (four states each) from those fp32
+//    rows, or, in verify and for fp32 inputs, straight from the TMA tile in
+//    the input dtype; groups of LPC steps are reduced across the LPC
 //    lanes of a channel with log2(LPC) shuffle rounds, each lane finishing one
 //    output y = (C.h + D*x) * silu(z), which goes to a shared-memory tile that
 //    one thread writes out with a TMA store.
@@ -43,6 +45,7 @@
 // conversion step each warp forms the dt tile of its own 8 channels with r/16
 // mma.sync m16n8k16 (fp32 accumulation), and its lanes convert the channel
 // pairs and steps that the accumulator layout gives them.
+#include <stddef.h>
 #include <string.h>
 
 #include "common.cuh"
@@ -66,11 +69,15 @@ constexpr int kPrefillStages = 4;  // TMA ring depth for long spans
 // or more dt_low boxes: one stage less keeps 4 CTAs per SM.
 constexpr int kPrefillStagesWide = 3;
 constexpr int kVerifyStages = 2;   // verify spans are short
+// Verify CTAs per SM the register budget must allow (5: 96 registers). The
+// scan reads its shared tiles through shared-state-space loads, which the
+// compiler may schedule ahead of the h_all stores; below 96 registers those
+// early loads spill.
 #ifndef MB_VERIFY_MINB
-#define MB_VERIFY_MINB 8   // verify CTAs per SM the register budget must allow (64 registers)
+#define MB_VERIFY_MINB 5
 #endif
 #ifndef MB_VERIFY_FUSED_MINB
-#define MB_VERIFY_FUSED_MINB 6   // the same with the Delta projection in the kernel (80 registers)
+#define MB_VERIFY_FUSED_MINB 5   // the same with the Delta projection in the kernel
 #endif
 
 // Lane geometry: LPC lanes share one channel, each holding kSPL states.
@@ -97,11 +104,27 @@ struct Conv {
     float2 xs[kT][CH];          // (D*x, silu(z)); silu(z) = 1 without a gate
 };
 
-template <typename T, int CH, int STAGES, bool kFuse>
+// B and C rows widened to fp32 once per chunk (bf16 prefill): the scan then
+// reads four states of each with one shared load and no per-lane conversion.
+// Verify spans are a single chunk, where the extra pass only lengthens the
+// critical path; they read the bf16 tiles directly.
+template <bool kWide>
+struct alignas(16) WideBC {
+    float B[kT][kDState];
+    float C[kT][kDState];
+};
+template <>
+struct WideBC<false> {};
+
+template <typename T, bool kStoreAll>
+constexpr bool kWideBC = sizeof(T) == 2 && !kStoreAll;
+
+template <typename T, int CH, int STAGES, bool kFuse, bool kWide>
 struct Smem {
     Raw<T, CH, kFuse> raw[STAGES];
     Conv<CH> cv[2];
-    T ys[2][kT][CH];            // output tiles, written out by TMA stores
+    WideBC<kWide> wbc[2];       // with cv: chunk i in slot i % 2
+    alignas(128) T ys[2][kT][CH];   // output tiles, written out by TMA stores
     uint64_t full[STAGES];
 };
 
@@ -131,8 +154,8 @@ __device__ __forceinline__ uint32_t swz(int row, int chunk) {
     return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
-template <typename T, int CH, int STAGES, bool kFuse>
-__device__ __forceinline__ void issue_chunk(Smem<T, CH, STAGES, kFuse> &s, const PrefillArgs &a, int stage,
+template <typename T, int CH, int STAGES, bool kFuse, bool kWide>
+__device__ __forceinline__ void issue_chunk(Smem<T, CH, STAGES, kFuse, kWide> &s, const PrefillArgs &a, int stage,
                                             int64_t chunk, int d0, int b, unsigned char *fz,
                                             uint32_t extra_bytes = 0) {
     constexpr uint32_t tok = kT * CH * sizeof(T), bc = kT * kDState * sizeof(T);
@@ -212,10 +235,12 @@ struct FuseCtx {
     int nks;           // dt_rank / 16
 };
 
-// Convert one chunk: raw TMA tiles -> fp32 (Delta, Delta*x), (D*x, silu z).
-template <typename T, int CH, bool kFuse>
-__device__ __forceinline__ void convert(Conv<CH> &cv, const Raw<T, CH, kFuse> &r, const ConvRole<CH> &cr,
-                                        int64_t t0, int64_t L, bool gate, const FuseCtx &fx) {
+// Convert one chunk: raw TMA tiles -> fp32 (Delta, Delta*x), (D*x, silu z)
+// and, with kWide, fp32 rows of B and C.
+template <typename T, int CH, bool kFuse, bool kWide>
+__device__ __forceinline__ void convert(Conv<CH> &cv, WideBC<kWide> &wbc, const Raw<T, CH, kFuse> &r,
+                                        const ConvRole<CH> &cr, int64_t t0, int64_t L, bool gate,
+                                        const FuseCtx &fx) {
     float acc[4];
     if constexpr (kFuse) project_delta<CH>(acc, fx.dtl, fx.w, fx.nks);
 #pragma unroll
@@ -240,6 +265,12 @@ __device__ __forceinline__ void convert(Conv<CH> &cv, const Raw<T, CH, kFuse> &r
         }
         *reinterpret_cast<float4 *>(&cv.dg[t][c]) = dg;
         *reinterpret_cast<float4 *>(&cv.xs[t][c]) = xs;
+    }
+    if constexpr (kWide) {   // thread (t, j): four states of B (j < 4) or C (j >= 4) at step t
+        static_assert(kThreads == kT * 8 && kDState == 16, "one quarter row of B or C per thread");
+        const int t = threadIdx.x >> 3, j = threadIdx.x & 7;
+        const float4 v = ld_quad(j < 4 ? &r.B[t][4 * j] : &r.C[t][4 * (j - 4)]);
+        *reinterpret_cast<float4 *>(j < 4 ? &wbc.B[t][4 * j] : &wbc.C[t][4 * (j - 4)]) = v;
     }
 }
 
@@ -278,10 +309,16 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
     constexpr int CH = G::kCh;
     static_assert(!kFuse || (LPC == 4 && sizeof(T) == 2 && CH == 8 * kWarps),
                   "the fused Delta projection maps one 8-channel mma tile per warp (bf16)");
-    using S = Smem<T, CH, STAGES, kFuse>;
+    constexpr bool kWide = kWideBC<T, kStoreAll>;
+    using S = Smem<T, CH, STAGES, kFuse, kWide>;
+    // every TMA source or destination in S starts on a 128-byte boundary
+    using R = Raw<T, CH, kFuse>;
+    static_assert(sizeof(R) % 128 == 0 && offsetof(R, z) % 128 == 0 && offsetof(R, B) % 128 == 0 &&
+                      offsetof(R, C) % 128 == 0 && offsetof(R, dt) % 128 == 0 && offsetof(S, raw) % 128 == 0 &&
+                      offsetof(S, ys) % 128 == 0 && (sizeof(T) * kT * CH) % 128 == 0,
+                  "TMA tiles must be 128-byte aligned");
     extern __shared__ unsigned char smem_dyn[];
-    S &s = *reinterpret_cast<S *>((reinterpret_cast<uintptr_t>(smem_dyn) + 127) &
-                                  ~static_cast<uintptr_t>(127));
+    S &s = smem_aligned<S>(smem_dyn);
     // fused Delta projection: dt_low stage boxes, then the W_dt boxes (1024-aligned)
     uint32_t fz_addr = 0;   // shared address of the first dt_low box
     unsigned char *fz = nullptr;
@@ -404,7 +441,7 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
         if constexpr (kFuse) f.dtl = fz_addr + (uint32_t)(st * a.nbox) * kDtlBox;
         return f;
     };
-    if (ok && nch > 0) convert(s.cv[0], s.raw[0], cr, c0 * kT, L, gate, stage_fx(0));
+    if (ok && nch > 0) convert(s.cv[0], s.wbc[0], s.raw[0], cr, c0 * kT, L, gate, stage_fx(0));
     if (__syncthreads_or(ok ? 0 : 1)) {
         if (tid == 0) {
             report(p.status, 4 /* MB_ERR_TIMEOUT */, 0);
@@ -420,7 +457,8 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
         const int nst = (int)((i + 1) % STAGES);
         ok = has_next ? mbar_wait(&s.full[nst], (uint32_t)(((i + 1) / STAGES) & 1)) : true;
         if constexpr (kFuse) ok = __all_sync(kFull, ok);
-        if (has_next && ok) convert(s.cv[(i + 1) & 1], s.raw[nst], cr, t0 + kT, L, gate, stage_fx(nst));
+        if (has_next && ok)
+            convert(s.cv[(i + 1) & 1], s.wbc[(i + 1) & 1], s.raw[nst], cr, t0 + kT, L, gate, stage_fx(nst));
 
         // (2) chunk i: decays of all kT steps, recurrence, shares of C.h
         if constexpr (kCkpt) {   // state before chunk i, for the backward's recompute
@@ -434,7 +472,8 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
             }
         }
         const Conv<CH> &cv = s.cv[i & 1];
-        const Raw<T, CH, kFuse> &rs = s.raw[i % STAGES];   // B, C straight from the TMA tile
+        const Raw<T, CH, kFuse> &rs = s.raw[i % STAGES];   // without kWide: B, C straight from the TMA tile
+        const WideBC<kWide> &wb = s.wbc[i & 1];
         float2 ab[kT][G::kPairs];
         float gx[kT];
 #pragma unroll
@@ -455,8 +494,14 @@ __global__ void __launch_bounds__(kThreads, kStoreAll ? (kFuse ? MB_VERIFY_FUSED
             float2 bp[G::kPairs], cp[G::kPairs];
 #pragma unroll
             for (int k = 0; k < G::kPairs; k += 2) {
-                const float4 b4 = ld_quad(&rs.B[t][G::kSPL * q + 2 * k]);
-                const float4 c4 = ld_quad(&rs.C[t][G::kSPL * q + 2 * k]);
+                float4 b4, c4;
+                if constexpr (kWide) {
+                    b4 = *reinterpret_cast<const float4 *>(&wb.B[t][G::kSPL * q + 2 * k]);
+                    c4 = *reinterpret_cast<const float4 *>(&wb.C[t][G::kSPL * q + 2 * k]);
+                } else {
+                    b4 = ld_quad(&rs.B[t][G::kSPL * q + 2 * k]);
+                    c4 = ld_quad(&rs.C[t][G::kSPL * q + 2 * k]);
+                }
                 bp[k] = make_float2(b4.x, b4.y); bp[k + 1] = make_float2(b4.z, b4.w);
                 cp[k] = make_float2(c4.x, c4.y); cp[k + 1] = make_float2(c4.z, c4.w);
             }
@@ -585,7 +630,7 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
         !make_map(&a.tm_C, p.C, bf16, p.batch, p.seqlen, kDState, kDState, p.bc_stride) ||
         !make_map(&a.tm_y, p.y, bf16, p.batch, p.seqlen, p.d_inner, kCh))
         return cudaErrorInvalidValue;
-    const size_t smem = sizeof(Smem<T, kCh, STAGES, kFuse>) + 128 + fuse_bytes;
+    const size_t smem = sizeof(Smem<T, kCh, STAGES, kFuse, kWideBC<T, kStoreAll>>) + 128 + fuse_bytes;
     const int64_t ctas = ((p.d_inner + kCh - 1) / kCh) * p.batch;   // per segment of L
     cudaError_t e;
     if constexpr (kSplittable) {

@@ -18,6 +18,16 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// The dynamic shared memory `dyn` (an extern __shared__ array) rounded up to
+// a 128-byte boundary and viewed as an S. The rounding is an offset added to
+// the array itself: a round trip through an integer would hide the shared
+// state space from the compiler, which then emits generic loads and stores
+// (64-bit addresses, a state-space check per access) for every use.
+template <typename S>
+__device__ __forceinline__ S &smem_aligned(unsigned char *dyn) {
+    return *reinterpret_cast<S *>(dyn + ((128u - (smem_u32(dyn) & 127u)) & 127u));
+}
+
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
 }

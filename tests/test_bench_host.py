@@ -86,3 +86,21 @@ def test_traffic_record_needs_matching_source(tmp_path, monkeypatch):
     (src / "k.cu").write_text("kernel source v2\n")
     assert bench.traffic_from_profiles("my_kernel") is None
     assert bench.traffic_from_profiles("other") is None
+
+
+def test_traffic_record_covers_every_listed_source(tmp_path, monkeypatch):
+    (tmp_path / "profiles").mkdir()
+    src = tmp_path / "paper_2401_13660_gb300" / "csrc"
+    src.mkdir(parents=True)
+    (src / "k.cu").write_text("kernel\n")
+    (src / "h.cuh").write_text("header v1\n")
+    import hashlib
+    sha = hashlib.sha256(b"kernel\nheader v1\n").hexdigest()[:16]
+    (tmp_path / "profiles" / "ncu_traffic.txt").write_text(
+        f"kernel=my_kernel source=k.cu,h.cuh sha={sha} bytes_per_launch=500 scale=2\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.traffic_from_profiles("my_kernel") == 1000.0
+    (src / "h.cuh").write_text("header v2\n")   # a header change also retires the record
+    assert bench.traffic_from_profiles("my_kernel") is None
+    (src / "h.cuh").unlink()
+    assert bench.traffic_from_profiles("my_kernel") is None
