@@ -16,8 +16,10 @@
 // 4q .. 4q+3 of channel warp*8 + c8. Chunks of kCkptSteps steps are taken in
 // reverse order through a ring of 3-D TMA tile loads (dt, x, z, dout, B, C).
 // Per chunk:
-//  * conversion (once per (t, channel pair)): Delta, Delta*x, x, dy into
-//    shared memory;
+//  * conversion (once per (t, channel pair)): Delta, Delta*x and dy into
+//    shared memory; for bf16 inputs also the chunk's B and C rows, widened
+//    to fp32 once instead of in every lane of both sweeps (x, needed only
+//    where a step is finished, is read there from the input tile);
 //  * recompute: from the chunk's checkpoint, the forward states of the 16
 //    steps (to shared memory, one float4 per lane and step) and each lane's
 //    share of C.h (for y);
@@ -35,6 +37,7 @@
 // conversion buffer and one dB/dC buffer, so that 4 CTAs fit on an SM.
 // dA, dD, dbias are accumulated in registers and added atomically at the end
 // (one contribution per batch row); dh0 is stored directly.
+#include <stddef.h>
 #include <string.h>
 
 #include "common.cuh"
@@ -59,14 +62,26 @@ struct BRaw {  // TMA destinations; member offsets are multiples of 128 B
     T C[kBT][kDState];
 };
 
+template <bool kWide>
 struct BConv {
-    float4 a[kBT][kBCh];   // (Delta, Delta*x, x, dy)
+    float2 dg[kBT][kBCh];   // (Delta, Delta*x)
+    float dy[kBT][kBCh];    // dJ/dy * silu(z)
+};
+// bf16 inputs: B and C rows widened to fp32 once per chunk (both sweeps read
+// four states of each per step; the space comes from keeping x out of the
+// conversion tile: the few readers of x take it from the input tile)
+template <>
+struct BConv<true> {
+    float2 dg[kBT][kBCh];
+    float dy[kBT][kBCh];
+    float B[kBT][kDState];
+    float C[kBT][kDState];
 };
 
 template <typename T>
 struct BSmem {
     BRaw<T> raw[kBStages];
-    BConv cv;
+    BConv<sizeof(T) == 2> cv;
     float4 hs[kBT][kBThreads];        // recomputed states of the chunk, per lane
     T gx[kBT][kBCh], gdt[kBT][kBCh], gz[kBT][kBCh];   // output tiles (TMA stores)
     float bc[kBT][32];   // per step: slot 8q + j, j < 4 dB[4q+j], else dC[4q+j-4]
@@ -117,31 +132,50 @@ __device__ __forceinline__ float sigmoid_v(float v) {
     return __fdividef(u, 1.f + u);
 }
 
-// Conversion of one chunk by one thread: channel pair cp at steps th, th + 8.
+// Conversion of one chunk by one thread: channel pair cp at steps th, th + 8
+// (and, for bf16, a quarter row of B or C).
 template <typename T>
-__device__ __forceinline__ void bconvert(BConv &cv, const BRaw<T> &r, int cp, int th, float2 bias, bool ok,
-                                         int64_t t0, int64_t L, bool gate) {
+__device__ __forceinline__ void bconvert(BConv<sizeof(T) == 2> &cv, const BRaw<T> &r, int cp, int th, float2 bias,
+                                         bool ok, int64_t t0, int64_t L, bool gate) {
 #pragma unroll
     for (int k = 0; k < kBT / 8; ++k) {
         const int t = th + 8 * k;
         const int c = 2 * cp;
-        float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f), a1 = a0;
+        float4 dg = make_float4(0.f, 0.f, 0.f, 0.f);   // (Delta, Delta*x) of channels c, c + 1
+        float2 dy = make_float2(0.f, 0.f);
         if (ok && t0 + t < L) {
             const float2 xv = ld_pair(&r.x[t][c]);
             const float2 dv = ld_pair(&r.dt[t][c]);
             const float2 ov = ld_pair(&r.dout[t][c]);
             const float d0 = softplus(dv.x + bias.x), d1 = softplus(dv.y + bias.y);   // as in the forward
-            float dy0 = ov.x, dy1 = ov.y;
+            dy = ov;
             if (gate) {
                 const float2 zv = ld_pair(&r.z[t][c]);
-                dy0 = ov.x * silu(zv.x);
-                dy1 = ov.y * silu(zv.y);
+                dy = make_float2(ov.x * silu(zv.x), ov.y * silu(zv.y));
             }
-            a0 = make_float4(d0, d0 * xv.x, xv.x, dy0);
-            a1 = make_float4(d1, d1 * xv.y, xv.y, dy1);
+            dg = make_float4(d0, d0 * xv.x, d1, d1 * xv.y);
         }
-        cv.a[t][c] = a0;
-        cv.a[t][c + 1] = a1;
+        *reinterpret_cast<float4 *>(&cv.dg[t][c]) = dg;
+        *reinterpret_cast<float2 *>(&cv.dy[t][c]) = dy;
+    }
+    if constexpr (sizeof(T) == 2) {   // thread (t, j): four states of B (j < 4) or C (j >= 4) at step t
+        static_assert(kBThreads == kBT * 8 && kDState == 16, "one quarter row of B or C per thread");
+        const int t = threadIdx.x >> 3, j = threadIdx.x & 7;
+        const float4 v = ld_quad(j < 4 ? &r.B[t][4 * j] : &r.C[t][4 * (j - 4)]);
+        *reinterpret_cast<float4 *>(j < 4 ? &cv.B[t][4 * j] : &cv.C[t][4 * (j - 4)]) = v;
+    }
+}
+
+// Four states of B and C at step t: the widened rows (bf16) or the tile (fp32).
+template <typename T>
+__device__ __forceinline__ void load_bc(const BConv<sizeof(T) == 2> &cv, const BRaw<T> &r, int t, int q,
+                                        float4 &b4, float4 &c4) {
+    if constexpr (sizeof(T) == 2) {
+        b4 = *reinterpret_cast<const float4 *>(&cv.B[t][4 * q]);
+        c4 = *reinterpret_cast<const float4 *>(&cv.C[t][4 * q]);
+    } else {
+        b4 = ld_quad(&r.B[t][4 * q]);
+        c4 = ld_quad(&r.C[t][4 * q]);
     }
 }
 
@@ -201,6 +235,14 @@ __device__ __forceinline__ void flush_bc(float (&bc)[kBT][32], const GradParams 
 template <typename T>
 __global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_constant__ BwdArgs a) {
     constexpr int S = kBStages;
+    using R = BRaw<T>;
+    using SM = BSmem<T>;
+    // every TMA source or destination starts on a 128-byte boundary
+    static_assert(sizeof(R) % 128 == 0 && offsetof(R, x) % 128 == 0 && offsetof(R, z) % 128 == 0 &&
+                      offsetof(R, dout) % 128 == 0 && offsetof(R, B) % 128 == 0 && offsetof(R, C) % 128 == 0 &&
+                      offsetof(SM, raw) % 128 == 0 && offsetof(SM, gx) % 128 == 0 &&
+                      offsetof(SM, gdt) % 128 == 0 && offsetof(SM, gz) % 128 == 0,
+                  "TMA tiles must be 128-byte aligned");
     extern __shared__ unsigned char smem_dyn[];
     BSmem<T> &s = smem_aligned<BSmem<T>>(smem_dyn);
     const ScanParams &p = a.p;
@@ -287,7 +329,7 @@ __global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_con
         }
 
         // (2) chunk i
-        const BConv &cv = s.cv;
+        const BConv<sizeof(T) == 2> &cv = s.cv;
         const BRaw<T> &rs = s.raw[j % S];
         const float2 hc[2] = {make_float2(ck_next.x, ck_next.y), make_float2(ck_next.z, ck_next.w)};
         if (i > 0) ck_next = load_ckpt(i - 1);
@@ -299,11 +341,11 @@ __global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_con
             float part[4];
 #pragma unroll
             for (int t = 0; t < kBT; ++t) {
-                const float4 av = cv.a[t][c];
+                const float2 av = cv.dg[t][c];
                 const float2 dd = make_float2(av.x, av.x), gg = make_float2(av.y, av.y);
                 const float2 e0 = mul2(dd, a2[0]), e1 = mul2(dd, a2[1]);
-                const float4 b4 = ld_quad(&rs.B[t][4 * q]);
-                const float4 c4 = ld_quad(&rs.C[t][4 * q]);
+                float4 b4, c4;
+                load_bc(cv, rs, t, q, b4, c4);
                 h0v = fma2(make_float2(ex2(e0.x), ex2(e0.y)), h0v, mul2(make_float2(b4.x, b4.y), gg));
                 h1v = fma2(make_float2(ex2(e1.x), ex2(e1.y)), h1v, mul2(make_float2(b4.z, b4.w), gg));
                 hs[t][tid] = make_float4(h0v.x, h0v.y, h1v.x, h1v.y);
@@ -318,13 +360,13 @@ __global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_con
         float4 hcur = hs[kBT - 1][tid];   // h_t; h_{t-1} is loaded each step
 #pragma unroll
         for (int t = kBT - 1; t >= 0; --t) {
-            const float4 av = cv.a[t][c];   // (Delta, Delta*x, x, dy)
+            const float2 av = cv.dg[t][c];   // (Delta, Delta*x)
             const float2 dd = make_float2(av.x, av.x), gx = make_float2(av.y, av.y);
-            const float2 dy = make_float2(av.w, av.w);
+            const float2 dy = make_float2(cv.dy[t][c], cv.dy[t][c]);
             const float2 e0 = mul2(dd, a2[0]), e1 = mul2(dd, a2[1]);
             const float2 ab0 = make_float2(ex2(e0.x), ex2(e0.y)), ab1 = make_float2(ex2(e1.x), ex2(e1.y));
-            const float4 b4 = ld_quad(&rs.B[t][4 * q]);
-            const float4 c4 = ld_quad(&rs.C[t][4 * q]);
+            float4 b4, c4;
+            load_bc(cv, rs, t, q, b4, c4);
             const float4 hprev = t > 0 ? hs[t - 1][tid] : make_float4(hc[0].x, hc[0].y, hc[1].x, hc[1].y);
             const float2 hp0 = make_float2(hprev.x, hprev.y), hp1 = make_float2(hprev.z, hprev.w);
             const float2 ht0 = make_float2(hcur.x, hcur.y), ht1 = make_float2(hcur.z, hcur.w);
@@ -349,8 +391,9 @@ __global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_con
                 const float S1 = reduce4(s1[0], s1[1], s1[2], s1[3], q);
                 const float S2 = reduce4(s2[0], s2[1], s2[2], s2[3], q);
                 const int tq = t + q;
-                const float4 aq = cv.a[tq][c];
                 const bool live = chan_ok && t0 + tq < L;
+                const float delta = cv.dg[tq][c].x, dyq = cv.dy[tq][c];
+                const float xq = live ? to_f32(rs.x[tq][c]) : 0.f;
                 const float sig = live ? sigmoid_v(to_f32(rs.dt[tq][c]) + dtb) : 0.f;
                 float qz = 0.f;
                 if (gate && live) {
@@ -358,10 +401,10 @@ __global__ void __launch_bounds__(kBThreads, 4) backward_kernel(const __grid_con
                     const float sz = __fdividef(1.f, 1.f + ex2(-zt * kLog2e));
                     qz = to_f32(rs.dout[tq][c]) * sz * fmaf(zt, 1.f - sz, 1.f);
                 }
-                const float dx = fmaf(aq.x, S1, aq.w * dsk);
-                const float ddt = fmaf(aq.z, S1, S2) * sig;
-                const float y = fmaf(dsk, aq.z, yv[t >> 2]);
-                dD_acc = fmaf(aq.w, aq.z, dD_acc);
+                const float dx = fmaf(delta, S1, dyq * dsk);
+                const float ddt = fmaf(xq, S1, S2) * sig;
+                const float y = fmaf(dsk, xq, yv[t >> 2]);
+                dD_acc = fmaf(dyq, xq, dD_acc);
                 db_acc += ddt;
                 store_out(s.gx, tq, c, dx);
                 store_out(s.gdt, tq, c, ddt);

@@ -266,11 +266,17 @@ __device__ __forceinline__ void convert(Conv<CH> &cv, WideBC<kWide> &wbc, const 
         *reinterpret_cast<float4 *>(&cv.dg[t][c]) = dg;
         *reinterpret_cast<float4 *>(&cv.xs[t][c]) = xs;
     }
-    if constexpr (kWide) {   // thread (t, j): four states of B (j < 4) or C (j >= 4) at step t
-        static_assert(kThreads == kT * 8 && kDState == 16, "one quarter row of B or C per thread");
-        const int t = threadIdx.x >> 3, j = threadIdx.x & 7;
-        const float4 v = ld_quad(j < 4 ? &r.B[t][4 * j] : &r.C[t][4 * (j - 4)]);
-        *reinterpret_cast<float4 *>(j < 4 ? &wbc.B[t][4 * j] : &wbc.C[t][4 * (j - 4)]) = v;
+    if constexpr (kWide) {   // item (t, j): four states of B (j < 4) or C (j >= 4) at step t
+        static_assert(kDState == 16, "quarter rows of B and C");
+        constexpr int kItems = kT * 8, kRounds = (kItems + kThreads - 1) / kThreads;
+#pragma unroll
+        for (int u = 0; u < kRounds; ++u) {
+            const int it = (int)threadIdx.x + u * kThreads;
+            if (kItems % kThreads != 0 && it >= kItems) break;
+            const int t = it >> 3, j = it & 7;
+            const float4 v = ld_quad(j < 4 ? &r.B[t][4 * j] : &r.C[t][4 * (j - 4)]);
+            *reinterpret_cast<float4 *>(j < 4 ? &wbc.B[t][4 * j] : &wbc.C[t][4 * (j - 4)]) = v;
+        }
     }
 }
 
