@@ -97,7 +97,9 @@ __device__ __forceinline__ float4 lds4(const __nv_bfloat16 *p) {
 // for the tile's 4 rows; lane q evaluates the channel scalars (Delta, Delta*x,
 // D*x, silu z) of row q only and shares Delta, Delta*x by shuffle, and after
 // the 4-lane reduction owns row q's output. New states go straight from
-// registers to global memory (512 contiguous bytes per warp and row).
+// registers to global memory (512 contiguous bytes per warp and row). The
+// round-robin order changes the channel block from tile to tile, so each
+// lane loads its channel's A row, dt_bias and D one tile ahead.
 // kResume (speculative decoding, after the bifurcation of Algorithm 1): row s
 // starts from h0[s] or h_all[s, accept[s]-1] instead of the state itself, so
 // the rollback needs no copy of its own; rows with an accept count outside
@@ -168,13 +170,31 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constan
     const int c = warp * 8 + g;
     float4 *state = reinterpret_cast<float4 *>(p.h_out);
     T *y = static_cast<T *>(p.y);
-    int64_t cur_d0 = -1;
-    float2 a01 = make_float2(0.f, 0.f), a23 = a01;
-    float bias = 0.f, dsk = 0.f;
+    // Channel constants (A row, dt_bias, D) of the next tile, loaded one tile
+    // ahead so that their latency overlaps the current tile.
+    float4 nav = make_float4(0.f, 0.f, 0.f, 0.f);
+    float nbias = 0.f, ndsk = 0.f;
+    auto load_const = [&](int k) {
+        nav = make_float4(0.f, 0.f, 0.f, 0.f);
+        nbias = ndsk = 0.f;
+        if (k < a.ntiles) {
+            const int64_t dn = (int64_t)(k % a.ntiles_d) * kStepCh + c;
+            if (dn < D) {
+                nav = ldg4(p.A + dn * kDState + 4 * q);
+                nbias = p.dt_bias ? __ldg(p.dt_bias + dn) : 0.f;
+                ndsk = p.D ? __ldg(p.D + dn) : 0.f;
+            }
+        }
+    };
+    load_const(blockIdx.x);
     for (int j = 0;; ++j) {
         const int k = blockIdx.x + j * gridDim.x;
         if (k >= a.ntiles) break;
         const int si = j % kStepStages;
+        const float2 a01 = make_float2(nav.x * kLog2e, nav.y * kLog2e);
+        const float2 a23 = make_float2(nav.z * kLog2e, nav.w * kLog2e);
+        const float bias = nbias, dsk = ndsk;
+        load_const(k + gridDim.x);
         if (!mbar_wait(&s.full[si], (uint32_t)((j / kStepStages) & 1))) {
             if (lane == 0) report(p.status, 4 /* MB_ERR_TIMEOUT */, k);
             break;
@@ -182,15 +202,6 @@ __global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constan
         const int64_t d0 = (int64_t)(k % a.ntiles_d) * kStepCh, b0 = (int64_t)(k / a.ntiles_d) * kStepRows;
         const int64_t d = d0 + c;
         const bool dok = d < D;
-        if (d0 != cur_d0) {
-            cur_d0 = d0;
-            const int64_t dd = dok ? d : 0;
-            const float4 av = ldg4(p.A + dd * kDState + 4 * q);
-            a01 = make_float2(av.x * kLog2e, av.y * kLog2e);
-            a23 = make_float2(av.z * kLog2e, av.w * kLog2e);
-            bias = (dok && p.dt_bias) ? __ldg(p.dt_bias + dd) : 0.f;
-            dsk = (dok && p.D) ? __ldg(p.D + dd) : 0.f;
-        }
         const StepStage<T> &t = s.st[si];
         float4 h[kStepRows];
 #pragma unroll
@@ -307,19 +318,43 @@ cudaError_t launch_step_typed(const ScanParams &p, const float *h_all, const int
         return cudaErrorInvalidValue;
     const size_t smem = sizeof(StepSmem<T>) + 128;
     auto kern = step_kernel<T, kResume>;
-    static int ctas = 0;   // resident CTAs per SM x SMs, computed once per process (per instantiation)
-    if (ctas == 0) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        int dev = 0, sms = 0, per = 0;
+    // Device limits, computed once per process (per instantiation): SMs,
+    // resident CTAs per SM, shared memory per SM and reserved per CTA.
+    static int sms = 0, per = 0;
+    static size_t smem_sm = 0, smem_reserved = 0, smem_optin = 0;
+    if (sms == 0) {
+        int dev = 0, n = 0, r = 0, sm_bytes = 0, rsv = 0, optin = 0;
+        cudaError_t e;
         if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, kern, kStepThreads, smem)) != cudaSuccess)
+        if ((e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess ||
+            (e = cudaDeviceGetAttribute(&sm_bytes, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev)) != cudaSuccess ||
+            (e = cudaDeviceGetAttribute(&rsv, cudaDevAttrReservedSharedMemoryPerBlock, dev)) != cudaSuccess ||
+            (e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess)
             return e;
-        ctas = sms * (per > 0 ? per : 1);
+        // the padded requests below stay within the opt-in maximum
+        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, optin)) != cudaSuccess)
+            return e;
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, kern, kStepThreads, smem)) != cudaSuccess)
+            return e;
+        smem_sm = (size_t)sm_bytes;
+        smem_reserved = (size_t)rsv;
+        smem_optin = (size_t)optin;
+        per = r > 0 ? r : 1;
+        sms = n > 0 ? n : 1;
     }
+    const int ctas = sms * per;
     const int grid = a.ntiles < ctas ? a.ntiles : ctas;
-    return launch_pdl(true, kern, dim3(grid), dim3(kStepThreads), smem, s, a);
+    // A grid of at most one wave needs only m = ceil(tiles / SMs) CTAs per SM.
+    // Left to the resident limit, the block scheduler stacks up to `per` of
+    // them on some SMs while others stay idle; asking for more than
+    // 1 / (m + 1) of an SM's shared memory per CTA spreads them instead.
+    size_t smem_launch = smem;
+    const int m = (grid + sms - 1) / sms;
+    if (m < per) {
+        const size_t spread = smem_sm / (size_t)(m + 1) - smem_reserved + 128;
+        if (spread > smem_launch && spread <= smem_optin) smem_launch = spread;
+    }
+    return launch_pdl(true, kern, dim3(grid), dim3(kStepThreads), smem_launch, s, a);
 }
 
 }  // namespace
