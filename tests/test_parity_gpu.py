@@ -266,3 +266,22 @@ def test_step_ragged_channel_count():
     y = _step(inp, state, 0)
     ry, rh, _ = oracle_scan(inp)
     assert rel_err(y, ry) <= TOL["bf16"] and rel_err(state, rh) <= TOL["bf16"]
+
+
+def test_step_rows_independent_of_the_launch_shape():
+    """The same rows stepped within grids of different shapes are bit-identical:
+    256 rows x 2048 channels (512 tiles: a persistent grid at the resident
+    limit), their first 32 rows (256 tiles: one wave spread at 2 CTAs per SM)
+    and first 4 rows (32 tiles: 1 CTA per SM). Checked against the oracle too."""
+    inp = make_inputs(256, 1, 2048, 16, "bf16", "normal", seed=53, device=DEV)
+    outs = {}
+    for rows in (256, 32, 4):
+        sub = {k: (v[:rows].contiguous() if torch.is_tensor(v) and v.shape[0] == 256 else v) for k, v in inp.items()}
+        state = sub["h0"].clone()
+        outs[rows] = (_step(sub, state, 0), state)
+    for rows in (32, 4):
+        assert torch.equal(outs[rows][0], outs[256][0][:rows])
+        assert torch.equal(outs[rows][1], outs[256][1][:rows])
+    small = {k: (v[:4].contiguous() if torch.is_tensor(v) and v.shape[0] == 256 else v) for k, v in inp.items()}
+    ry, rh, _ = oracle_scan(small)
+    assert rel_err(outs[4][0], ry) <= TOL["bf16"] and rel_err(outs[4][1], rh) <= TOL["bf16"]
