@@ -662,12 +662,12 @@ cudaError_t launch_typed(const ScanParams &p, cudaStream_t s) {
 }  // namespace
 
 // Time split: only when the batch rows and channel tiles give at most one CTA
-// per SM (a CTA alone on an SM runs a chunk in ~1.1 us, four together take
-// ~2 us each: the SM idles); then into as many segments as fill the resident
-// slots (4 per SM for bf16 at 118 registers, 3 for fp32), each at least
-// kMinSegChunks chunks long. The summary pass costs ~70 % of a scan, so at 1.7
-// CTAs per SM (batch 4 x 2048 channels) the split measured slower (677 -> 766 us)
-// while batch 1 x 2048 channels x 8192 steps went 554 -> 212 us.
+// per SM (a CTA alone on an SM leaves most of its issue slots idle); then into
+// as many segments as fill the resident slots (4 per SM for bf16, 3 for fp32),
+// each at least kMinSegChunks chunks long. The summary pass repeats most of a
+// scan, so at 1.7 CTAs per SM (batch 4 x 2048 channels) the split measured
+// slower (604 -> 653 us) while batch 1 x 2048 channels x 8192 steps went
+// 480 -> 180 us.
 constexpr int64_t kMinSegChunks = 8;
 
 int64_t prefill_segments(const ScanParams &p, bool bf16) {
