@@ -7,9 +7,12 @@
 // states (64 contiguous bytes). In the step kernel four lanes share a channel,
 // each holding 4 states in one float4, so a warp moves 512 contiguous bytes
 // of state per instruction.
-#include "common.cuh"
 #include <string.h>
 
+#include <atomic>
+#include <mutex>
+
+#include "common.cuh"
 #include "tma.cuh"
 
 namespace mbscan {
@@ -318,30 +321,47 @@ cudaError_t launch_step_typed(const ScanParams &p, const float *h_all, const int
         return cudaErrorInvalidValue;
     const size_t smem = sizeof(StepSmem<T>) + 128;
     auto kern = step_kernel<T, kResume>;
-    // Device limits, computed once per process (per instantiation): SMs,
-    // resident CTAs per SM, shared memory per SM and reserved per CTA.
-    static int sms = 0, per = 0;
-    static size_t smem_sm = 0, smem_reserved = 0, smem_optin = 0;
-    if (sms == 0) {
-        int dev = 0, n = 0, r = 0, sm_bytes = 0, rsv = 0, optin = 0;
-        cudaError_t e;
-        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-        if ((e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess ||
-            (e = cudaDeviceGetAttribute(&sm_bytes, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev)) != cudaSuccess ||
-            (e = cudaDeviceGetAttribute(&rsv, cudaDevAttrReservedSharedMemoryPerBlock, dev)) != cudaSuccess ||
-            (e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess)
-            return e;
-        // the padded requests below stay within the opt-in maximum
-        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, optin)) != cudaSuccess)
-            return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, kern, kStepThreads, smem)) != cudaSuccess)
-            return e;
-        smem_sm = (size_t)sm_bytes;
-        smem_reserved = (size_t)rsv;
-        smem_optin = (size_t)optin;
-        per = r > 0 ? r : 1;
-        sms = n > 0 ? n : 1;
+    // Device limits, computed once per device (per instantiation) and published
+    // through `ready`: SMs, resident CTAs per SM, shared memory per SM and
+    // reserved per CTA.
+    struct Limits {
+        std::atomic<int> ready;
+        int sms, per;
+        size_t smem_sm, smem_reserved, smem_optin;
+    };
+    constexpr int kMaxDevices = 64;
+    static Limits lim[kMaxDevices];
+    static std::mutex init_mu;
+    int dev = 0;
+    cudaError_t e;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    Limits &l = lim[dev];
+    if (!l.ready.load(std::memory_order_acquire)) {
+        std::lock_guard<std::mutex> guard(init_mu);
+        if (!l.ready.load(std::memory_order_relaxed)) {
+            int n = 0, r = 0, sm_bytes = 0, rsv = 0, optin = 0;
+            if ((e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess ||
+                (e = cudaDeviceGetAttribute(&sm_bytes, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev)) !=
+                    cudaSuccess ||
+                (e = cudaDeviceGetAttribute(&rsv, cudaDevAttrReservedSharedMemoryPerBlock, dev)) != cudaSuccess ||
+                (e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess)
+                return e;
+            // the padded requests below stay within the opt-in maximum
+            if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, optin)) != cudaSuccess)
+                return e;
+            if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, kern, kStepThreads, smem)) != cudaSuccess)
+                return e;
+            l.sms = n > 0 ? n : 1;
+            l.per = r > 0 ? r : 1;
+            l.smem_sm = (size_t)sm_bytes;
+            l.smem_reserved = (size_t)rsv;
+            l.smem_optin = (size_t)optin;
+            l.ready.store(1, std::memory_order_release);
+        }
     }
+    const int sms = l.sms, per = l.per;
+    const size_t smem_sm = l.smem_sm, smem_reserved = l.smem_reserved, smem_optin = l.smem_optin;
     const int ctas = sms * per;
     const int grid = a.ntiles < ctas ? a.ntiles : ctas;
     // A grid of at most one wave needs only m = ceil(tiles / SMs) CTAs per SM.

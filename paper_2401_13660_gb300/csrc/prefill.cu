@@ -48,6 +48,8 @@
 #include <stddef.h>
 #include <string.h>
 
+#include <atomic>
+
 #include "common.cuh"
 #include "tma.cuh"
 
@@ -673,18 +675,18 @@ constexpr int64_t kMinSegChunks = 8;
 int64_t prefill_segments(const ScanParams &p, bool bf16) {
     if (p.batch <= 0 || p.d_inner <= 0 || p.seqlen <= 0 || p.dt_low) return 1;
     constexpr int kMaxDevices = 64;
-    static int sm_count[kMaxDevices] = {0};   // per device, filled on first use
+    static std::atomic<int> sm_count[kMaxDevices];   // per device, filled on first use (0: not yet)
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 1;
-    if (sm_count[dev] == 0) {
-        int v = 0;
-        if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) return 1;
-        sm_count[dev] = v;
+    int sms = sm_count[dev].load(std::memory_order_relaxed);
+    if (sms == 0) {
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) return 1;
+        sm_count[dev].store(sms, std::memory_order_relaxed);   // every writer stores the same value
     }
     constexpr int kCh = Geom<kPrefillLanesPerChannel>::kCh;
-    const int64_t slots = (int64_t)sm_count[dev] * (bf16 ? 4 : 3);
+    const int64_t slots = (int64_t)sms * (bf16 ? 4 : 3);
     const int64_t ctas = p.batch * ((p.d_inner + kCh - 1) / kCh);
-    if (ctas > sm_count[dev]) return 1;
+    if (ctas > sms) return 1;
     const int64_t nchunks = (p.seqlen + kT - 1) / kT;
     int64_t nseg = slots / ctas;
     if (nseg > nchunks / kMinSegChunks) nseg = nchunks / kMinSegChunks;
