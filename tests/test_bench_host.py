@@ -1,5 +1,7 @@
-"""CPU checks of bench.py's host logic: algorithmic byte counts and the
-multi-rank timing reduction (two gloo ranks on 127.0.0.1)."""
+"""CPU checks of bench.py's host logic: algorithmic byte counts, the
+multi-rank timing reduction (two gloo ranks on 127.0.0.1) and the JSON line
+of the oracle (reference) arm, alone and under torchrun with two ranks."""
+import json
 import os
 import socket
 
@@ -9,6 +11,8 @@ import torch.distributed as dist
 import torch.multiprocessing as mp
 
 import bench
+
+ROOT_DIR = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 def test_algorithmic_bytes_of_the_workloads():
@@ -104,3 +108,45 @@ def test_traffic_record_covers_every_listed_source(tmp_path, monkeypatch):
     assert bench.traffic_from_profiles("my_kernel") is None
     (src / "h.cuh").unlink()
     assert bench.traffic_from_profiles("my_kernel") is None
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _reference_cmd():
+    import sys
+    return [sys.executable, os.path.join(ROOT_DIR, "bench.py"), "--impl", "reference", "--steps", "1",
+            "--warmup", "3", "--ref-fraction", str(1 / 128)]
+
+
+def test_reference_arm_prints_the_contract_line():
+    """The oracle arm (no GPU) prints one JSON line with the contract's keys."""
+    import subprocess
+    r = subprocess.run(_reference_cmd(), capture_output=True, text=True, timeout=900, cwd=ROOT_DIR)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == "GB/s"
+    assert d["value"] > 0 and d["steps"] == 1 and d["warmup"] == 3 and d["n_gpus"] == 1
+    assert d["higher_is_better"] is True and d["vs_baseline"] is None
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
+    assert d["e2e"]["value"] == d["value"] and d["config"]["workload"] == bench.WORKLOAD_NAME
+
+
+def test_reference_arm_under_two_ranks_prints_once():
+    """Under torchrun with 2 ranks, rank 0 alone runs and prints; both exit 0."""
+    import subprocess
+    import sys
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(_free_port())] + _reference_cmd()[1:] + ["--gpus", "2"]
+    r = subprocess.run(cmd, capture_output=True, text=True, timeout=900, cwd=ROOT_DIR)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.lstrip().startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0].strip())
+    assert d["impl"] == "reference" and d["n_gpus"] == 2
