@@ -107,8 +107,9 @@ __device__ __forceinline__ float4 lds4(const __nv_bfloat16 *p) {
 // starts from h0[s] or h_all[s, accept[s]-1] instead of the state itself, so
 // the rollback needs no copy of its own; rows with an accept count outside
 // [0, k] are reported and left untouched.
+// Minimum CTAs per SM: those its shared memory allows (3 for bf16, 2 for fp32).
 template <typename T, bool kResume>
-__global__ void __launch_bounds__(kStepThreads) step_kernel(const __grid_constant__ StepArgs a) {
+__global__ void __launch_bounds__(kStepThreads, sizeof(T) == 2 ? 3 : 2) step_kernel(const __grid_constant__ StepArgs a) {
     extern __shared__ unsigned char smem_dyn[];
     StepSmem<T> &s = smem_aligned<StepSmem<T>>(smem_dyn);
     const ScanParams &p = a.p;
