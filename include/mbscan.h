@@ -26,7 +26,7 @@
  *    A failed launch returns MB_ERR_CUDA.
  *  - Outputs must not alias inputs unless stated.
  *  - Supported today: d_state == 16, dtype MB_F32 or MB_BF16,
- *    d_inner % 8 == 0, batch*seqlen*d_inner < 2^31.
+ *    d_inner % 8 == 0, batch*seqlen*d_inner <= 2^31.
  */
 #ifndef MBSCAN_H
 #define MBSCAN_H
@@ -200,6 +200,12 @@ mb_status mb_accept_topk(const void *logits, int32_t dtype, const uint8_t *draft
  * `state` [batch, d_inner, d_state] fp32 is read and updated in place; y is
  * [batch, 1, d_inner]. Used for the corrector loop of Algorithm 1 and for
  * plain generation.
+ *   ws, ws_bytes : workspace (at least 256 bytes, 256-byte aligned, its
+ *                  status block zeroed once after allocation) or NULL. The
+ *                  kernel's waits for its own TMA copies are bounded; one that
+ *                  gives up records MB_ERR_TIMEOUT there (read it with
+ *                  mb_check), and the rows it did not reach keep their old
+ *                  state. With ws == NULL such a timeout is not reported.
  * Launch overlap: the step kernel is launched with programmatic dependent
  * launch. It waits for the previous kernel on the stream to complete before
  * touching memory, and lets the next kernel launch while it runs. A kernel
@@ -208,7 +214,7 @@ mb_status mb_accept_topk(const void *logits, int32_t dtype, const uint8_t *draft
  * before reading y or state, as CUDA requires for any such launch. Plainly
  * launched work is ordered as usual.
  */
-mb_status mb_step(const mb_scan_args *args, float *state, void *stream);
+mb_status mb_step(const mb_scan_args *args, float *state, void *ws, size_t ws_bytes, void *stream);
 
 /*
  * Resume after the bifurcation (Algorithm 1): one recurrent decode step for
@@ -347,20 +353,24 @@ mb_status mb_selftest_timeout(void *ws, size_t ws_bytes, int64_t wait_cycles, vo
  * library; the paper has no counterpart.)
  *
  * Some callers cannot allocate device memory at the point where they run the
- * scan: code recorded into a CUDA graph or running under an allocator that
- * owns all device memory, real-time paths that must not allocate after
- * start-up, or plugins that are handed only input and output buffers. This
- * entry point computes exactly what mb_scan_prefill computes, for the same
- * arguments, but its scratch (the status block of bounded device-side
- * waits, 256 bytes) is a fixed array inside the library, one per GPU, kept
- * for as long as the library is loaded. It calls no allocator.
+ * scan: code running under an allocator that owns all device memory,
+ * real-time paths that must not allocate after start-up, or plugins that are
+ * handed only their input and output buffers. This entry point takes the
+ * same arguments as mb_scan_prefill but no workspace: its scratch (the
+ * 256-byte status block of the bounded device-side waits) is a fixed array
+ * inside the library, one per GPU, kept for as long as the library is
+ * loaded. It calls no allocator.
  *
  *  - Arguments, layouts and h_last rules are those of mb_scan_prefill.
- *  - A problem whose workspace would exceed the fixed 256-byte array is
- *    rejected with MB_ERR_UNSUPPORTED before anything is launched (no
- *    supported shape needs more today).
- *  - The first call on each GPU looks up the array's device address with that
- *    GPU current; make that first call outside any stream capture.
+ *  - The fixed array has room for the status block only (256 bytes), not for
+ *    the segment summaries of the time split, so every span runs unsplit:
+ *    the result is bit for bit that of mb_scan_prefill given a 256-byte
+ *    workspace. (A single long prompt therefore takes the unsplit kernel's
+ *    time; mb_scan_prefill with mb_workspace_size(args) bytes is faster.)
+ *  - The first call on each GPU looks up the array's device address with
+ *    that GPU current and keeps it for the life of the process; make that
+ *    first call before any stream capture, and do not call this entry point
+ *    again on a device after resetting it (cudaDeviceReset).
  *  - Every call clears the array on `stream` before the launch. All calls on
  *    one GPU share the one array, so calls that may run at the same time on
  *    the GPU (different streams without ordering) race on it; order them.

@@ -163,6 +163,29 @@ mb_status setup_split(const mb_scan_args *args, ScanParams &p, const float *h_la
 
 mb_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MB_OK : MB_ERR_CUDA; }
 
+// The prefill's rules for h_last (shared by mb_scan_prefill and
+// mb_scan_prefill_noalloc): 16-byte aligned; it may be exactly h0 (in-place
+// resume) but must not partially overlap h0, nor overlap y or any input that
+// the kernel still reads while it writes h_last.
+mb_status check_h_last(const mb_scan_args *args, const float *h_last) {
+    if (!h_last) return MB_OK;
+    if (!aligned16(h_last)) return MB_ERR_INVALID_ARG;
+    const int64_t sbytes = args->batch * args->d_inner * args->d_state * 4;
+    const Range rh = range_of(h_last, sbytes);
+    if (args->h0 != h_last && overlap(rh, range_of(args->h0, sbytes))) return MB_ERR_INVALID_ARG;
+    const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
+    const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
+    const int64_t bc = bc_bytes(args);
+    const Range others[] = {range_of(args->y, tok), range_of(args->x, tok), range_of(args->dt, tok),
+                            range_of(args->z, tok), range_of(args->B, bc), range_of(args->C, bc),
+                            range_of(args->A, args->d_inner * args->d_state * 4),
+                            range_of(args->D, args->d_inner * 4), range_of(args->dt_bias, args->d_inner * 4),
+                            range_of(args->dt_low, dtl_bytes(args)), range_of(args->W_dt, wdt_bytes(args))};
+    for (const Range &r : others)
+        if (overlap(rh, r)) return MB_ERR_INVALID_ARG;
+    return MB_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -179,20 +202,7 @@ mb_status mb_scan_prefill(const mb_scan_args *args, float *h_last, void *ws, siz
     mb_status st = check_args(args, false);
     if (st != MB_OK) return st;
     if ((st = check_ws(args, ws, ws_bytes)) != MB_OK) return st;
-    const int64_t sbytes = args->batch * args->d_inner * args->d_state * 4;
-    if (h_last) {
-        if (!aligned16(h_last)) return MB_ERR_INVALID_ARG;
-        const Range rh = range_of(h_last, sbytes);
-        // h_last may be exactly h0 (in-place resume) but not partially overlap it.
-        if (args->h0 != h_last && overlap(rh, range_of(args->h0, sbytes))) return MB_ERR_INVALID_ARG;
-        const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
-        const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
-        if (overlap(rh, range_of(args->y, tok)) || overlap(rh, range_of(args->x, tok)) ||
-            overlap(rh, range_of(args->dt, tok)) || overlap(rh, range_of(args->z, tok)) ||
-            overlap(rh, range_of(args->dt_low, dtl_bytes(args))) ||
-            overlap(rh, range_of(args->W_dt, wdt_bytes(args))))
-            return MB_ERR_INVALID_ARG;
-    }
+    if ((st = check_h_last(args, h_last)) != MB_OK) return st;
     if (args->batch * args->d_inner == 0) return MB_OK;
     ScanParams p = to_params(args, h_last, static_cast<StatusBlock *>(ws));
     const bool bf16 = args->dtype == MB_BF16;
@@ -293,13 +303,15 @@ mb_status mb_accept_topk(const void *logits, int32_t dtype, const uint8_t *draft
                                            (cudaStream_t)stream));
 }
 
-mb_status mb_step(const mb_scan_args *args, float *state, void *stream) {
+mb_status mb_step(const mb_scan_args *args, float *state, void *ws, size_t ws_bytes, void *stream) {
     mb_status st = check_args(args, true);
     if (st != MB_OK) return st;
     if (args->dt_low) return MB_ERR_UNSUPPORTED;   // the step kernel takes dt
     const int64_t chans = args->batch * args->d_inner;
     if (chans == 0) return MB_OK;
     if (state == nullptr || !aligned16(state)) return MB_ERR_INVALID_ARG;
+    if (ws && ((reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < mbscan::kStatusBytes))
+        return MB_ERR_INVALID_ARG;
     const Range rs = range_of(state, chans * args->d_state * 4);
     const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
     const int64_t tok = chans * es;
@@ -307,10 +319,13 @@ mb_status mb_step(const mb_scan_args *args, float *state, void *stream) {
                             range_of(args->dt, tok), range_of(args->B, bc_bytes(args)),
                             range_of(args->C, bc_bytes(args)),
                             range_of(args->A, args->d_inner * args->d_state * 4),
-                            range_of(args->dt_low, dtl_bytes(args)), range_of(args->W_dt, wdt_bytes(args))};
+                            range_of(args->D, args->d_inner * 4), range_of(args->dt_bias, args->d_inner * 4),
+                            range_of(args->dt_low, dtl_bytes(args)), range_of(args->W_dt, wdt_bytes(args)),
+                            range_of(ws, ws ? (int64_t)mbscan::kStatusBytes : 0)};
     for (const Range &r : others)
         if (overlap(rs, r)) return MB_ERR_INVALID_ARG;
-    ScanParams p = to_params(args, state, nullptr);
+    if (ws && overlap(range_of(ws, mbscan::kStatusBytes), range_of(args->y, tok))) return MB_ERR_INVALID_ARG;
+    ScanParams p = to_params(args, state, static_cast<StatusBlock *>(ws));
     p.h0 = nullptr;
     return from_cuda(mbscan::launch_step(p, args->dtype == MB_BF16, (cudaStream_t)stream));
 }
@@ -524,19 +539,22 @@ const char *mb_version(void) { return "mbscan 0.1.0 sm_103a"; }
 // ---------------------------------------------------------------------------
 // Allocation-free prefill (mb_scan_prefill_noalloc).
 //
-// The prefill kernel needs a small block of device scratch (the status block
-// that its bounded waits write). Normally the caller provides it as `ws`. For
+// The prefill kernel needs a small block of device scratch: the status block
+// that its bounded waits write. Normally the caller provides it as `ws`. For
 // callers that may not allocate device memory, this file owns one fixed
 // scratch array per device instead: a file-scope __device__ array of
-// kNoAllocScratchBytes. Host code must never hand the array's name to a
-// kernel (on the host it is only a stand-in symbol); its device address is
-// looked up once per device with cudaGetSymbolAddress while that device is
-// current, and that address is what the kernel receives. The array lives for
-// as long as the library is loaded on the device and keeps the previous
-// call's contents, so every call clears it first on its stream.
+// kNoAllocScratchBytes (the 256-byte status block, nothing more). Host code
+// must never hand the array's name to a kernel (on the host it is only a
+// stand-in symbol); its device address is looked up once per device with
+// cudaGetSymbolAddress while that device is current, and that address is what
+// the kernel receives. The array lives for as long as the library is loaded
+// on the device and keeps the previous call's contents, so every call clears
+// it first on its stream. The array holds no room for the segment summaries
+// of the time split, so every span runs unsplit: exactly what mb_scan_prefill
+// does when its workspace is 256 bytes.
 namespace {
 
-constexpr size_t kNoAllocScratchBytes = 256;   // the largest workspace it can stand in for
+constexpr size_t kNoAllocScratchBytes = mbscan::kStatusBytes;
 constexpr int kNoAllocMaxDevices = 64;
 
 }  // namespace
@@ -549,7 +567,8 @@ std::mutex g_noalloc_mutex;
 void *g_noalloc_addr[kNoAllocMaxDevices];   // device address of the array, per device
 
 // Device address of g_noalloc_scratch on the current device, looked up on
-// the first call for that device.
+// the first call for that device and kept for the life of the process (the
+// primary context of that device is assumed to live as long).
 mb_status noalloc_scratch(void **out) {
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess) return MB_ERR_CUDA;
@@ -565,34 +584,18 @@ mb_status noalloc_scratch(void **out) {
     return MB_OK;
 }
 
-// Same checks on h_last as mb_scan_prefill.
-mb_status check_h_last(const mb_scan_args *args, const float *h_last) {
-    if (!h_last) return MB_OK;
-    if (!aligned16(h_last)) return MB_ERR_INVALID_ARG;
-    const int64_t sbytes = args->batch * args->d_inner * args->d_state * 4;
-    const Range rh = range_of(h_last, sbytes);
-    if (args->h0 != h_last && overlap(rh, range_of(args->h0, sbytes))) return MB_ERR_INVALID_ARG;
-    const int64_t es = args->dtype == MB_BF16 ? 2 : 4;
-    const int64_t tok = args->batch * args->seqlen * args->d_inner * es;
-    if (overlap(rh, range_of(args->y, tok)) || overlap(rh, range_of(args->x, tok)) ||
-        overlap(rh, range_of(args->dt, tok)) || overlap(rh, range_of(args->z, tok)))
-        return MB_ERR_INVALID_ARG;
-    return MB_OK;
-}
-
 }  // namespace
 
 extern "C" mb_status mb_scan_prefill_noalloc(const mb_scan_args *args, float *h_last, void *stream) {
     mb_status st = check_args(args, false);
     if (st != MB_OK) return st;
     if ((st = check_h_last(args, h_last)) != MB_OK) return st;
-    const size_t need = mb_workspace_size(args);
-    if (need > kNoAllocScratchBytes) return MB_ERR_UNSUPPORTED;   // larger than the fixed scratch
     if (args->batch * args->d_inner == 0) return MB_OK;
     void *scratch = nullptr;
     if ((st = noalloc_scratch(&scratch)) != MB_OK) return st;
     cudaStream_t s = (cudaStream_t)stream;
-    if (need > 0 && cudaMemsetAsync(scratch, 0, need, s) != cudaSuccess) return MB_ERR_CUDA;
+    if (cudaMemsetAsync(scratch, 0, kNoAllocScratchBytes, s) != cudaSuccess) return MB_ERR_CUDA;
+    // p.nseg stays 1 (to_params): the span runs unsplit
     ScanParams p = to_params(args, h_last, static_cast<StatusBlock *>(scratch));
     return from_cuda(mbscan::launch_prefill(p, args->dtype == MB_BF16, s));
 }

@@ -74,7 +74,7 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
             lib.mb_scan_prefill.argtypes = [ap, vp, vp, sz, vp]
             lib.mb_scan_verify.argtypes = [ap, vp, vp, sz, vp]
             lib.mb_rollback.argtypes = [vp, vp, vp, vp, i64, i64, i64, i64, vp, vp]
-            lib.mb_step.argtypes = [ap, vp, vp]
+            lib.mb_step.argtypes = [ap, vp, vp, sz, vp]
             lib.mb_check.argtypes = [vp, vp, ctypes.POINTER(i64)]
             lib.mb_accept_topk.argtypes = [vp, ctypes.c_int32, vp, i64, i64, ctypes.c_int32, vp, vp]
             lib.mb_step_resume.argtypes = [ap, vp, vp, i64, vp, vp, sz, vp]
@@ -274,13 +274,16 @@ def mb_rollback(h0, h_all, accept, h_out, *, ws=None, stream=None):
     return h_out
 
 
-def mb_step(x, dt, B, C, A, y, state, *, z=None, D=None, dt_bias=None, stream=None, dt_low=None,
+def mb_step(x, dt, B, C, A, y, state, *, z=None, D=None, dt_bias=None, ws=None, stream=None, dt_low=None,
             W_dt=None):
     """One decode step: x, dt, z, y [batch, 1, d_inner]; B, C [batch, 1, d_state];
-    state [batch, d_inner, d_state] updated in place."""
+    state [batch, d_inner, d_state] updated in place. ws (optional, >= 256
+    bytes): status block where a timed-out wait is recorded (mb_check)."""
     a = make_args(x, dt, B, C, A, y, z=z, D=D, dt_bias=dt_bias, dt_low=dt_low, W_dt=W_dt)
     _need(state, "state", torch.float32, (a.batch, a.d_inner, a.d_state), x.device)
-    rc = load_library().mb_step(ctypes.byref(a), _ptr(state), _stream(stream))
+    _need(ws, "ws", torch.uint8, None, x.device)
+    nbytes = 0 if ws is None else ws.numel()
+    rc = load_library().mb_step(ctypes.byref(a), _ptr(state), _ptr(ws), nbytes, _stream(stream))
     _check(rc, "mb_step")
     return y, state
 

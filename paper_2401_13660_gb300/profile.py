@@ -48,8 +48,8 @@ def algorithmic_bytes(entry: str, w, s_in: int) -> int:
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--entry", choices=["prefill", "verify", "rollback", "step", "backward", "decode_model",
-                                        "write_floor"], required=True)
+    ap.add_argument("--entry", choices=["prefill", "verify", "rollback", "step", "backward", "decode_model"],
+                    required=True)
     ap.add_argument("--workload", required=True,
                     help="a workload of inputs.WORKLOADS, or for --entry decode_model a decoder.CONFIGS name")
     ap.add_argument("--batch", type=int, default=256, help="streams of --entry decode_model")
@@ -59,8 +59,6 @@ def main():
     dev = torch.device("cuda:0")
     if a.entry == "decode_model":
         return decode_model(a, dev)
-    if a.entry == "write_floor":
-        return write_floor(a, dev)
     w = WORKLOADS[a.workload]
     mb.load_library()
     nsets = a.layers if a.entry == "step" else 1
@@ -135,32 +133,6 @@ def main():
     nbytes = algorithmic_bytes(a.entry, w, 2 if w.dtype == "bf16" else 4)
     print(json.dumps({"entry": a.entry, "workload": w.name, "iters": a.iters, "us_per_launch": round(us, 3),
                       "algorithmic_bytes": nbytes, "GB/s": round(nbytes / (us * 1e-6) / 1e9, 1)}))
-
-
-def write_floor(a, dev):
-    """Device time to write, from nothing, a buffer the size of the workload's
-    per-position states (verify's h_all): a PyTorch fill after a 256 MB write
-    that leaves L2 full of dirty lines, as the kernels before a verify do. No
-    library kernel runs; this is the hardware's rate for that write stream,
-    the floor under verify's h_all bytes."""
-    w = WORKLOADS[a.workload]
-    buf = torch.empty(w.batch * w.seqlen * w.d_inner * N_STATE, dtype=torch.float32, device=dev)
-    flush = torch.empty(64 << 20, dtype=torch.float32, device=dev)
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-    times = []
-    for i in range(a.iters + 3):
-        flush.fill_(float(i))
-        ev[0].record()
-        buf.fill_(float(i))
-        ev[1].record()
-        torch.cuda.synchronize()
-        if i >= 3:
-            times.append(1e3 * ev[0].elapsed_time(ev[1]))
-    nb = buf.numel() * 4
-    best, mean = min(times), sum(times) / len(times)
-    print(json.dumps({"entry": "write_floor", "workload": w.name, "iters": a.iters, "bytes": nb,
-                      "us_best": round(best, 3), "us_mean": round(mean, 3),
-                      "GB/s_best": round(nb / (best * 1e-6) / 1e9, 1)}))
 
 
 def decode_model(a, dev):

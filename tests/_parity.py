@@ -5,9 +5,15 @@ import torch
 
 import oracle
 
-# Tolerances on err = max |g - r| / max(|r|, rms(r)) per output tensor: the
-# state is fp32 in both cases; bf16 inputs/outputs add the bf16 rounding of y.
+# Tolerances on err = max |g - r| / max(|r|, rms(r)) per output tensor. TOL is
+# the bar for y: 1e-4 with fp32 inputs, 2e-2 with bf16 inputs (y is rounded to
+# bf16, 2^-9 relative, and inherits that rounding through D*x and the gate).
+# TOL_STATE is the bar for the fp32 states (h_last, h_all, the stepped state):
+# they are never rounded to bf16, so with bf16 inputs (widened exactly on both
+# sides) only fp32 arithmetic separates them from the oracle (about 1e-5
+# measured); 1e-3 still flags a state error 100x smaller than the y bar.
 TOL = {"f32": 1e-4, "bf16": 2e-2}
+TOL_STATE = {"f32": 1e-4, "bf16": 1e-3}
 
 
 def rel_err(got, ref) -> float:

@@ -112,7 +112,7 @@ def test_zero_sized_calls_launch_nothing():
     lib = mb.load_library()
     assert _prefill(_args(batch=0)) == mb.MB_OK
     assert _call("mb_scan_verify", _args(L=0), None, FAKE + (200 << 32), 256, None) == mb.MB_OK
-    assert _call("mb_step", _args(batch=0, L=1), None, None) == mb.MB_OK
+    assert _call("mb_step", _args(batch=0, L=1), None, None, 0, None) == mb.MB_OK
     assert lib.mb_rollback(None, None, None, None, 0, 16, 64, 16, None, None) == mb.MB_OK
 
 
@@ -121,10 +121,15 @@ def test_verify_and_step_checks():
     assert _call("mb_scan_verify", a, None, FAKE + (200 << 32), 256, None) == mb.MB_ERR_INVALID_ARG
     assert _call("mb_scan_verify", a, a.h0, FAKE + (200 << 32), 256, None) == mb.MB_ERR_INVALID_ARG
     s = _args(L=2)
-    assert _call("mb_step", s, FAKE + (210 << 32), None) == mb.MB_ERR_INVALID_ARG   # seqlen != 1
+    assert _call("mb_step", s, FAKE + (210 << 32), None, 0, None) == mb.MB_ERR_INVALID_ARG   # seqlen != 1
     s = _args(L=1)
-    assert _call("mb_step", s, None, None) == mb.MB_ERR_INVALID_ARG
-    assert _call("mb_step", s, s.x, None) == mb.MB_ERR_INVALID_ARG               # state aliases x
+    assert _call("mb_step", s, None, None, 0, None) == mb.MB_ERR_INVALID_ARG
+    assert _call("mb_step", s, s.x, None, 0, None) == mb.MB_ERR_INVALID_ARG      # state aliases x
+    st = FAKE + (210 << 32)
+    assert _call("mb_step", s, st, FAKE + (200 << 32) + 16, 256, None) == mb.MB_ERR_INVALID_ARG  # ws not 256-aligned
+    assert _call("mb_step", s, st, FAKE + (200 << 32), 128, None) == mb.MB_ERR_INVALID_ARG       # ws too small
+    assert _call("mb_step", s, st, st, 256, None) == mb.MB_ERR_INVALID_ARG                       # ws inside state
+    assert _call("mb_step", s, st, s.y, 256, None) == mb.MB_ERR_INVALID_ARG                      # ws overlaps y
 
 
 def test_rollback_checks():
@@ -262,7 +267,7 @@ def test_fused_delta_checks():
     assert lib.mb_scan_prefill_ckpt(ctypes.byref(_fused(L=40)), None, FAKE + (40 << 32), ws, 256,
                                     None) == mb.MB_ERR_UNSUPPORTED   # the training path takes dt
     s = _fused(L=1)
-    assert _call("mb_step", s, FAKE + (210 << 32), None) == mb.MB_ERR_UNSUPPORTED   # the step takes dt
+    assert _call("mb_step", s, FAKE + (210 << 32), None, 0, None) == mb.MB_ERR_UNSUPPORTED   # the step takes dt
     acc = FAKE + (220 << 32)
     assert lib.mb_step_resume(ctypes.byref(s), FAKE + (230 << 32), acc, 4, FAKE + (210 << 32), None, 0,
                               None) == mb.MB_ERR_UNSUPPORTED
@@ -316,3 +321,24 @@ def test_verify_resume_checks():
     b.y = prev                                                # y overlaps h_all_prev
     assert call(args=b) == mb.MB_ERR_INVALID_ARG
     assert call(args=_args(batch=0, L=8)) == mb.MB_OK
+
+
+def test_noalloc_prefill_host_checks():
+    # mb_scan_prefill_noalloc applies mb_scan_prefill's argument and h_last
+    # rules before it touches the GPU (here: before any CUDA call at all).
+    lib = mb.load_library()
+    f = lib.mb_scan_prefill_noalloc
+    f.argtypes = [ctypes.POINTER(mb.mb_scan_args), ctypes.c_void_p, ctypes.c_void_p]
+    f.restype = ctypes.c_int
+    assert f(ctypes.byref(_args(batch=0)), None, None) == mb.MB_OK
+    a = _fused()
+    assert f(ctypes.byref(a), a.dt_low, None) == mb.MB_ERR_INVALID_ARG        # h_last overlaps dt_low
+    assert f(ctypes.byref(a), a.W_dt, None) == mb.MB_ERR_INVALID_ARG          # h_last overlaps W_dt
+    a = _args()
+    assert f(ctypes.byref(a), a.h0 + 16, None) == mb.MB_ERR_INVALID_ARG       # partial overlap with h0
+    assert f(ctypes.byref(a), a.B, None) == mb.MB_ERR_INVALID_ARG             # h_last overlaps B
+    assert f(ctypes.byref(a), a.x + 4, None) == mb.MB_ERR_INVALID_ARG         # misaligned
+    assert _prefill(_fused(), h_last=_fused().dt_low) == mb.MB_ERR_INVALID_ARG
+    assert _prefill(_args(), h_last=_args().B) == mb.MB_ERR_INVALID_ARG
+    # valid arguments: without a GPU the call then fails at its first CUDA call
+    assert f(ctypes.byref(_args()), FAKE + (230 << 32), None) in (mb.MB_OK, mb.MB_ERR_CUDA)

@@ -13,7 +13,7 @@ from paper_2401_13660_gb300 import mbscan as mb
 from paper_2401_13660_gb300.inputs import make_inputs
 
 import oracle
-from _parity import TOL, oracle_scan, rel_err, to_np
+from _parity import TOL, TOL_STATE, oracle_scan, rel_err, to_np
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -35,14 +35,14 @@ def test_prefill_and_verify_general_a(dtype):
     mb.mb_scan_prefill(inp["x"], inp["dt"], inp["B"], inp["C"], inp["A"], y, z=inp["z"], D=inp["D"],
                        dt_bias=inp["dt_bias"], h0=inp["h0"], h_last=hl)
     ry, rh, rall = oracle_scan(inp, want_h_all=True)
-    assert rel_err(y, ry) <= TOL[dtype] and rel_err(hl, rh) <= TOL[dtype]
+    assert rel_err(y, ry) <= TOL[dtype] and rel_err(hl, rh) <= TOL_STATE[dtype]
     for L in (16, 37):   # single-chunk and multi-chunk verify spans
         sub = {k: (v[:, :L].contiguous() if k in ("x", "z", "dt", "B", "C") else v) for k, v in inp.items()}
         yv = torch.empty_like(sub["x"])
         h_all = torch.empty(3, L, 8 * 67, 16, device=DEV)
         mb.mb_scan_verify(sub["x"], sub["dt"], sub["B"], sub["C"], sub["A"], yv, h_all, z=sub["z"], D=sub["D"],
                           dt_bias=sub["dt_bias"], h0=sub["h0"])
-        assert rel_err(yv, ry[:, :L]) <= TOL[dtype] and rel_err(h_all, rall[:, :L]) <= TOL[dtype]
+        assert rel_err(yv, ry[:, :L]) <= TOL[dtype] and rel_err(h_all, rall[:, :L]) <= TOL_STATE[dtype]
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
@@ -57,7 +57,7 @@ def test_step_and_resume_general_a(dtype):
                    inp["C"][:, sl].contiguous(), inp["A"], y, state, z=inp["z"][:, sl].contiguous(), D=inp["D"],
                    dt_bias=inp["dt_bias"])
         assert rel_err(y, ry[:, sl]) <= TOL[dtype]
-    assert rel_err(state, rall[:, 2]) <= TOL[dtype]
+    assert rel_err(state, rall[:, 2]) <= TOL_STATE[dtype]
     # resume: verify the first 5 bytes, keep a per-stream prefix, step byte 5 from it
     span = {k: (v[:, :5].contiguous() if k in ("x", "z", "dt", "B", "C") else v) for k, v in inp.items()}
     yv = torch.empty_like(span["x"])
@@ -75,7 +75,7 @@ def test_step_and_resume_general_a(dtype):
         one = lambda k: to_np(nxt[k][s:s + 1])
         wy, wh, _ = oracle.scan(one("x"), one("dt"), one("B"), one("C"), to_np(inp["A"]), z=one("z"),
                                 D=to_np(inp["D"]), dt_bias=to_np(inp["dt_bias"]), h0=start)
-        assert rel_err(y[s:s + 1], wy) <= TOL[dtype] and rel_err(out[s:s + 1], wh) <= TOL[dtype]
+        assert rel_err(y[s:s + 1], wy) <= TOL[dtype] and rel_err(out[s:s + 1], wh) <= TOL_STATE[dtype]
 
 
 def test_backward_general_a():
@@ -105,4 +105,4 @@ def test_fused_delta_prefill_general_a():
     mb.mb_scan_prefill(inp["x"], None, inp["B"], inp["C"], inp["A"], y, z=inp["z"], D=inp["D"],
                        dt_bias=inp["dt_bias"], h0=inp["h0"], h_last=hl, dt_low=inp["dt_low"], W_dt=inp["W_dt"])
     ry, rh, _ = oracle_scan(inp)
-    assert rel_err(y, ry) <= TOL["bf16"] and rel_err(hl, rh) <= TOL["bf16"]
+    assert rel_err(y, ry) <= TOL["bf16"] and rel_err(hl, rh) <= TOL_STATE["bf16"]

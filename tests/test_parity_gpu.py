@@ -13,7 +13,7 @@ import oracle
 from paper_2401_13660_gb300 import mbscan as mb
 from paper_2401_13660_gb300.inputs import WORKLOADS, make_inputs, torch_dtype, workload_inputs
 
-from _parity import TOL, oracle_channels, oracle_scan, rel_err, to_np
+from _parity import TOL, TOL_STATE, oracle_channels, oracle_scan, rel_err, to_np
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -55,7 +55,7 @@ def test_prefill_tiny_fp32_full():
     y, hl = _prefill(inp)
     ry, rh, _ = oracle_scan(inp)
     assert rel_err(y, ry) <= TOL["f32"]
-    assert rel_err(hl, rh) <= TOL["f32"]
+    assert rel_err(hl, rh) <= TOL_STATE["f32"]
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
@@ -67,7 +67,7 @@ def test_prefill_ragged(dtype, shape, h0):
     y, hl = _prefill(inp)
     ry, rh, _ = oracle_scan(inp)
     assert rel_err(y, ry) <= TOL[dtype]
-    assert rel_err(hl, rh) <= TOL["f32" if dtype == "f32" else "bf16"]
+    assert rel_err(hl, rh) <= TOL_STATE["f32" if dtype == "f32" else "bf16"]
 
 
 def test_prefill_optional_operands_absent():
@@ -76,7 +76,7 @@ def test_prefill_optional_operands_absent():
     inp["dt_bias"] = None
     y, hl = _prefill(inp)
     ry, rh, _ = oracle_scan(inp)
-    assert rel_err(y, ry) <= TOL["f32"] and rel_err(hl, rh) <= TOL["f32"]
+    assert rel_err(y, ry) <= TOL["f32"] and rel_err(hl, rh) <= TOL_STATE["f32"]
     y2, _ = _prefill(inp, h_last=False)
     torch.testing.assert_close(y2, y, rtol=0, atol=0)
 
@@ -95,7 +95,7 @@ def test_prefill_h_last_in_place_over_h0():
     y = torch.empty_like(inp["x"])
     mb.mb_scan_prefill(inp["x"], inp["dt"], inp["B"], inp["C"], inp["A"], y, z=inp["z"],
                        D=inp["D"], dt_bias=inp["dt_bias"], h0=h, h_last=h)
-    assert rel_err(h, rh) <= TOL["f32"]
+    assert rel_err(h, rh) <= TOL_STATE["f32"]
 
 
 @pytest.mark.parametrize("name", ["mambabyte353m_prefill_b8_L8192", "mambabyte972m_prefill_b4_L8192"])
@@ -116,7 +116,7 @@ def test_prefill_full_size_sampled(name):
     gy = y.index_select(0, r_t)[:, :, c_t]
     gh = hl.index_select(0, r_t)[:, c_t]
     assert rel_err(gy, ry) <= TOL["bf16"]
-    assert rel_err(gh, rh) <= TOL["bf16"]
+    assert rel_err(gh, rh) <= TOL_STATE["bf16"]
 
 
 def test_prefill_split_equals_one_scan():
@@ -153,7 +153,7 @@ def test_prefill_a_zero_linear_growth():
     _, hl = _prefill(inp)
     delta = torch.nn.functional.softplus((inp["dt"][0, 0] + inp["dt_bias"]).double())
     want = inp["h0"][0].double() + L * (delta * inp["x"][0, 0].double())[:, None] * inp["B"][0, 0].double()[None]
-    assert rel_err(hl[0], want.cpu().numpy()) <= TOL["f32"]
+    assert rel_err(hl[0], want.cpu().numpy()) <= TOL_STATE["f32"]
 
 
 # ------------------------------------------------------------------ verify + rollback
@@ -163,7 +163,7 @@ def test_verify_full_size_against_oracle():
     y, h_all = _verify(inp)
     ry, rh, rall = oracle_scan(inp, want_h_all=True)
     assert rel_err(y, ry) <= TOL["bf16"]
-    assert rel_err(h_all, rall) <= TOL["bf16"]
+    assert rel_err(h_all, rall) <= TOL_STATE["bf16"]
     # rollback at the seeded accept counts: an index gather, bit-exact
     h_out = torch.empty_like(inp["h0"])
     mb.mb_rollback(inp["h0"], h_all, inp["accept"], h_out)
@@ -172,7 +172,7 @@ def test_verify_full_size_against_oracle():
                        h_all[torch.arange(w.batch, device=DEV), (acc - 1).clamp(min=0)])
     assert torch.equal(h_out, want)
     ro = oracle.rollback(to_np(inp["h0"]), rall, to_np(inp["accept"]).astype(np.int32))
-    assert rel_err(h_out, ro) <= TOL["bf16"]
+    assert rel_err(h_out, ro) <= TOL_STATE["bf16"]
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
@@ -180,7 +180,7 @@ def test_verify_matches_prefill_and_oracle_small(dtype):
     inp = make_inputs(5, 23, 40, 16, dtype, "normal", seed=31, device=DEV)
     y, h_all = _verify(inp)
     ry, _, rall = oracle_scan(inp, want_h_all=True)
-    assert rel_err(y, ry) <= TOL[dtype] and rel_err(h_all, rall) <= TOL[dtype]
+    assert rel_err(y, ry) <= TOL[dtype] and rel_err(h_all, rall) <= TOL_STATE[dtype]
     yp, hl = _prefill(inp)
     if dtype == "f32":
         torch.testing.assert_close(y, yp, rtol=1e-5, atol=1e-5)
@@ -189,9 +189,9 @@ def test_verify_matches_prefill_and_oracle_small(dtype):
 
 @pytest.mark.parametrize("dtype,L", [("bf16", 5), ("f32", 16), ("bf16", 1)])
 def test_verify_single_chunk_ragged_stays_in_bounds(dtype, L):
-    """Spans of at most one chunk stage the per-position states in shared
-    memory and write them with one tile store per CTA: positions past L and
-    channels past d_inner (536 = 16 full 32-channel tiles + 24) must be clipped,
+    """Spans of at most one chunk stream every per-position state from the
+    lanes' registers to h_all: positions past L and channels past d_inner
+    (536 = 16 full 32-channel tiles + 24) must be skipped,
     so a sentinel tail after h_all stays untouched and every stream's rows
     match the oracle."""
     b, D = 3, 8 * 67
@@ -204,7 +204,7 @@ def test_verify_single_chunk_ragged_stays_in_bounds(dtype, L):
                       D=inp.get("D"), dt_bias=inp.get("dt_bias"), h0=inp.get("h0"))
     ry, _, rall = oracle_scan(inp, want_h_all=True)
     assert torch.isnan(big[n:]).all()
-    assert rel_err(y, ry) <= TOL[dtype] and rel_err(h_all, rall) <= TOL[dtype]
+    assert rel_err(y, ry) <= TOL[dtype] and rel_err(h_all, rall) <= TOL_STATE[dtype]
 
 
 def test_rollback_edges_and_alias():
@@ -244,7 +244,7 @@ def test_step_full_size_one_layer():
     y = _step(inp, state, 0)
     ry, rh, _ = oracle_scan(inp)
     assert rel_err(y, ry) <= TOL["bf16"]
-    assert rel_err(state, rh) <= TOL["bf16"]
+    assert rel_err(state, rh) <= TOL_STATE["bf16"]
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
@@ -255,7 +255,7 @@ def test_steps_equal_one_scan(dtype):
     state = inp["h0"].clone()
     ys = [_step(inp, state, t) for t in range(12)]
     assert rel_err(torch.cat(ys, 1), ry) <= TOL[dtype]
-    assert rel_err(state, rh) <= TOL[dtype]
+    assert rel_err(state, rh) <= TOL_STATE[dtype]
     _, hl = _prefill(inp)
     torch.testing.assert_close(state, hl, rtol=1e-5, atol=1e-6)
 
@@ -265,7 +265,7 @@ def test_step_ragged_channel_count():
     state = inp["h0"].clone()
     y = _step(inp, state, 0)
     ry, rh, _ = oracle_scan(inp)
-    assert rel_err(y, ry) <= TOL["bf16"] and rel_err(state, rh) <= TOL["bf16"]
+    assert rel_err(y, ry) <= TOL["bf16"] and rel_err(state, rh) <= TOL_STATE["bf16"]
 
 
 def test_step_rows_independent_of_the_launch_shape():
@@ -284,4 +284,4 @@ def test_step_rows_independent_of_the_launch_shape():
         assert torch.equal(outs[rows][1], outs[256][1][:rows])
     small = {k: (v[:4].contiguous() if torch.is_tensor(v) and v.shape[0] == 256 else v) for k, v in inp.items()}
     ry, rh, _ = oracle_scan(small)
-    assert rel_err(outs[4][0], ry) <= TOL["bf16"] and rel_err(outs[4][1], rh) <= TOL["bf16"]
+    assert rel_err(outs[4][0], ry) <= TOL["bf16"] and rel_err(outs[4][1], rh) <= TOL_STATE["bf16"]

@@ -12,7 +12,7 @@ import torch
 from paper_2401_13660_gb300 import mbscan as mb
 from paper_2401_13660_gb300.inputs import make_inputs
 
-from _parity import TOL, oracle_channels, oracle_scan, rel_err
+from _parity import TOL, TOL_STATE, oracle_channels, oracle_scan, rel_err
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -41,7 +41,7 @@ def test_split_prefill_against_oracle(dtype, b, L, Dn, h0):
     assert n > 256   # these spans are split
     y, hl = _prefill(inp, ws)
     ry, rh, _ = oracle_scan(inp)
-    assert rel_err(y, ry) <= TOL[dtype] and rel_err(hl, rh) <= TOL[dtype]
+    assert rel_err(y, ry) <= TOL[dtype] and rel_err(hl, rh) <= TOL_STATE[dtype]
     assert mb.mb_check(ws) == (mb.MB_OK, -1)
     ws1, _ = _ws(inp, split=False)
     y1, hl1 = _prefill(inp, ws1)   # unsplit: the same values up to fp32 reassociation
@@ -61,7 +61,7 @@ def test_split_batch1_prompt_prefill_sampled():
     chans = [0, 31, 32, 1000, 2047]
     ry, rh, _ = oracle_channels(inp, [0], chans)
     c_t = torch.tensor(chans, device=DEV)
-    assert rel_err(y[:, :, c_t], ry) <= TOL["bf16"] and rel_err(hl[:, c_t], rh) <= TOL["bf16"]
+    assert rel_err(y[:, :, c_t], ry) <= TOL["bf16"] and rel_err(hl[:, c_t], rh) <= TOL_STATE["bf16"]
     ws1, _ = _ws(inp, split=False)
     y1, hl1 = _prefill(inp, ws1)
     assert rel_err(hl, hl1.double().cpu().numpy()) <= 1e-4
