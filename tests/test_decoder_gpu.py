@@ -10,7 +10,7 @@ import oracle
 from paper_2401_13660_gb300 import mbscan as mb
 from paper_2401_13660_gb300.decoder import CONFIGS, WEIGHT_KEYS, Decoder
 
-from _parity import rel_err, to_np
+from _parity import TOL, TOL_STATE, rel_err, to_np
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -126,21 +126,26 @@ def _oracle_decode_layerwise(dec, tokens_seq):
 
 def test_decoder_full_size_matches_oracle():
     """The 48-layer d_model 2304 decoder that bench.py times, at batch 2 over
-    two bytes, against the fp64 oracle.
+    two bytes, against the fp64 oracle, in three ways:
 
-    Both sides round to bf16 at the same tensor boundaries, but the GEMMs
-    accumulate in fp32 on the GPU and in fp64 in the oracle, so a value can
-    round to a neighbouring bf16 number (2^-8 relative). Over 48 layers such
-    flips compound through the residual stream: with fp32 accumulation
-    emulated on the host and no GPU at all, per-layer states drift from the
-    fp64 ones by up to 0.2 of their rms at layer 47. So every block step is
-    checked on the GPU's own inputs to that block (its residual, the previous
-    block's output and the states the GPU carried in), where only one block's
-    rounding separates the two sides (the same emulation stays within 1.2e-2),
-    and the logits of the whole decode are checked end to end. Bar 2e-2. The
-    traced eager pass is also checked bit for bit against the CUDA-graph
-    replay that the benchmark times."""
+    * each library kernel of every block on the exact tensors the GPU handed
+      it (traced): mb_rmsnorm, mb_conv1d_step, and mb_step whose new SSM state
+      is held to the fp32-state bar (1e-3) and y to 2e-2;
+    * every whole block step (oracle.block_step) on the GPU's inputs to that
+      block: block output, convolution window and residual;
+    * the logits of the whole two-byte decode, end to end.
+    The block-level and end-to-end bars are 2e-2: both sides round to bf16 at
+    the same tensor boundaries, but the GEMMs accumulate in fp32 on the GPU and
+    in fp64 in the oracle, so a value can land on a neighbouring bf16 number
+    (2^-8 relative), and such flips feed the scan's inputs. Through one block
+    they move the new SSM state by a few percent of its rms at worst (which is
+    why the state is checked on the scan's exact inputs); over 48 layers they
+    compound (a host-only emulation with fp32 accumulation drifts by up to 0.2
+    at layer 47), so nothing is compared after compounding except the logits.
+    The traced eager pass is checked bit for bit against the CUDA-graph replay
+    that the benchmark times."""
     cfg = CONFIGS["mambabyte_48x2304"]
+    R, N = cfg.dt_rank, cfg.d_state
     dec = Decoder(cfg, batch=2, device=DEV, seed=1)
     ref = Decoder(cfg, batch=2, device=DEV, seed=1, weights=(dec.layers, dec.emb, dec.norm_f))
     ref.capture()
@@ -157,16 +162,29 @@ def test_decoder_full_size_matches_oracle():
     ref.check()
     for a, b in zip(dec.ssm + dec.conv, ref.ssm + ref.conv):
         assert torch.equal(a, b)
-    worst = {"ssm": 0.0, "conv": 0.0, "out": 0.0, "residual": 0.0}
+    kern = {"rmsnorm": 0.0, "conv_out": 0.0, "step_y": 0.0, "step_state": 0.0}
+    block = {"residual": 0.0, "out": 0.0, "conv": 0.0}
     for l, L in enumerate(dec.layers):
         layer = {k: to_np(L[k]) for k in WEIGHT_KEYS}
         for tr in traces:
-            b = tr[l]
-            r, out, ssm, conv = oracle.block_step(layer, to_np(b["residual"]), to_np(b["add"]), to_np(b["ssm"]),
-                                                  to_np(b["conv"]), eps=cfg.eps)
-            for k, want in (("residual", r), ("out", out), ("ssm", ssm), ("conv", conv)):
-                worst[k] = max(worst[k], rel_err(b[k if k == "out" else k + "_out"], want))
-    assert worst["residual"] <= 1e-6 and max(worst.values()) <= 2e-2, worst
+            b = {k: to_np(v) for k, v in tr[l].items()}
+            # the library kernels on their exact inputs
+            _, hn = oracle.rmsnorm(b["residual"], layer["norm_w"], cfg.eps, b["add"])
+            kern["rmsnorm"] = max(kern["rmsnorm"], rel_err(tr[l]["h"], hn))
+            xc, cst = oracle.conv1d_step(b["conv"], b["x"], layer["conv_w"], layer["conv_b"])
+            assert np.array_equal(b["conv_out"], cst)
+            kern["conv_out"] = max(kern["conv_out"], rel_err(tr[l]["xc"], xc))
+            y, st = oracle.step(b["ssm"], x=b["xc"], dt=b["dt"], B=b["xdbl"][:, R:R + N], C=b["xdbl"][:, R + N:],
+                                A=layer["A"], z=b["z"], D=layer["D"], dt_bias=layer["dt_bias"])
+            kern["step_y"] = max(kern["step_y"], rel_err(tr[l]["y"], y))
+            kern["step_state"] = max(kern["step_state"], rel_err(tr[l]["ssm_out"], st))
+            # the whole block on the GPU's inputs to it
+            r, out, _, conv = oracle.block_step(layer, b["residual"], b["add"], b["ssm"], b["conv"], eps=cfg.eps)
+            for k, want in (("residual", r), ("out", out), ("conv", conv)):
+                block[k] = max(block[k], rel_err(tr[l][k if k == "out" else k + "_out"], want))
+    assert kern["rmsnorm"] <= 1e-2 and kern["conv_out"] <= 1e-2, kern
+    assert kern["step_y"] <= TOL["bf16"] and kern["step_state"] <= TOL_STATE["bf16"], kern
+    assert block["residual"] <= 1e-6 and block["out"] <= 2e-2 and block["conv"] <= 2e-2, block
     want, _, _ = _oracle_decode_layerwise(dec, seq)
     for gl, wl in zip(got, want):
         assert rel_err(gl, wl) <= 2e-2
