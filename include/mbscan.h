@@ -326,6 +326,35 @@ mb_status mb_conv1d_step(const void *x, void *state, const float *w, const float
                          int64_t batch, int64_t width, int32_t dtype, void *stream);
 
 /*
+ * The convolution step above fused with the x-projection that follows it
+ * (Figure 6; Table 6 "Pre-SSM 1D convolution" and "Delta, B, C from input
+ * x"), for decoding a whole model:
+ *   xc  = the output of mb_conv1d_step (same arithmetic, window updated the same way)
+ *   out[b, n] = sum_d xc[b, d] W[n, d]   ([dt_low | B | C] = xc W^T)
+ * with xc rounded to bf16 before the product (as the unfused pair does),
+ * products accumulated in fp32 and out rounded to bf16 once. The sum runs
+ * in width / 128 fp32 partial sums (one per 128 channels) added in a fixed
+ * order, so results are reproducible run to run and differ from one fp32
+ * GEMM only by rounding order.
+ *   x, xc  : [batch, width] bf16; xc is written
+ *   state  : [batch, 3, width] bf16, read and written (as mb_conv1d_step)
+ *   w, bias: [width, 4] fp32, [width] fp32 or NULL
+ *   W      : [n_out, width] bf16 (rows dt_low, then B, then C)
+ *   out    : [batch, n_out] bf16
+ *   dtype  : MB_BF16 only (MB_ERR_UNSUPPORTED otherwise)
+ *   ws     : 256-byte aligned, ws_bytes >= mb_conv_xproj_workspace_size(
+ *            batch, width, n_out): the status block, then the partial sums.
+ *            A wait for the W tile that gives up records MB_ERR_TIMEOUT there.
+ * Supported: width % 128 == 0, n_out in {40, 96, 144, 176} (dt_rank + 32
+ * for d_state 16 and dt_rank 8, 64, 112, 144); MB_ERR_UNSUPPORTED otherwise.
+ * xc, out, state and ws must not overlap one another or the inputs.
+ */
+size_t mb_conv_xproj_workspace_size(int64_t batch, int64_t width, int32_t n_out);
+mb_status mb_conv_xproj(const void *x, void *state, const float *w, const float *bias, const void *W, void *xc,
+                        void *out, int64_t batch, int64_t width, int32_t n_out, int32_t dtype, void *ws,
+                        size_t ws_bytes, void *stream);
+
+/*
  * Read and clear the status block of a workspace (blocking: waits for
  * `stream`). Returns MB_OK, or the first device-side error recorded by
  * calls on that workspace since the last mb_check. If detail != NULL it

@@ -82,10 +82,11 @@ __device__ __forceinline__ float2 ldg2(const __nv_bfloat16 *p) {
 // once every prerequisite grid has completed and its writes are visible, so
 // only shared-memory set-up overlaps the predecessor. pdl_trigger() lets the
 // next kernel launch before this one completes (it still waits for it). Only
-// the persistent decode step issues it: a grid of many short-lived CTAs that
-// triggers early lets the next grid's CTAs take SM slots as they free up,
-// which leaves SMs unevenly loaded when that grid fills less than every slot
-// (measured: back-to-back prefills of 448 CTAs, 822 -> 990 us).
+// the persistent decode step and the single-wave fused convolution +
+// x-projection issue it: a grid of many short-lived CTAs that triggers early
+// lets the next grid's CTAs take SM slots as they free up, which leaves SMs
+// unevenly loaded when that grid fills less than every slot (measured:
+// back-to-back prefills of 448 CTAs, 822 -> 990 us).
 #ifndef MB_PDL
 #define MB_PDL 1
 #endif
@@ -101,9 +102,10 @@ __device__ __forceinline__ void pdl_trigger() {
 }
 
 // Launch `kern` on `s`; with overlap = true it may start during the previous
-// kernel's tail (see pdl_wait). Only the decode step uses the overlap: next to
-// cuBLAS kernels (which trigger early) the short element-wise kernels measured
-// slower with it (whole-model decode 3.32 -> 3.38 ms), so they launch plainly.
+// kernel's tail (see pdl_wait). The decode step and the fused convolution +
+// x-projection with its reduction use the overlap (whole-model decode 2.92 ->
+// 2.89 ms); next to cuBLAS kernels (which trigger early) the short element-wise
+// kernels measured slower with it (3.32 -> 3.38 ms), so they launch plainly.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(bool overlap, void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
                        Args &&...args) {

@@ -91,6 +91,13 @@ cudaError_t launch_rmsnorm(const void *add, float *residual, const float *w, flo
                            int64_t batch, int64_t width, bool bf16, cudaStream_t s);
 cudaError_t launch_conv_step(const void *x, void *state, const float *w, const float *bias, void *out,
                              int64_t batch, int64_t width, bool bf16, cudaStream_t s);
+// Decode-step convolution fused with the x-projection (xproj.cu): supported
+// widths and output widths, the fp32 partial-sum scratch it needs, the launch.
+bool conv_xproj_supported(int64_t width, int n_out);
+size_t conv_xproj_partial_bytes(int64_t batch, int64_t width, int n_out);
+cudaError_t launch_conv_xproj(const void *x, void *state, const float *w, const float *bias, const void *W,
+                              void *xc, void *out, int64_t batch, int64_t width, int n_out, float *part,
+                              StatusBlock *status, cudaStream_t s);
 cudaError_t launch_step(const ScanParams &p, bool bf16, cudaStream_t s);
 // One step from the state kept after accept[s] drafted bytes: p.h0 (may be
 // null = zeros) when accept[s] == 0, else h_all[s, accept[s]-1]; the new state

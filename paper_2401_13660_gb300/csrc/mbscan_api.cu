@@ -498,6 +498,41 @@ mb_status mb_conv1d_step(const void *x, void *state, const float *w, const float
                                               (cudaStream_t)stream));
 }
 
+size_t mb_conv_xproj_workspace_size(int64_t batch, int64_t width, int32_t n_out) {
+    if (batch < 0 || batch > kMaxTokens || !mbscan::conv_xproj_supported(width, n_out)) return 0;
+    return mbscan::kStatusBytes + mbscan::conv_xproj_partial_bytes(batch, width, n_out);
+}
+
+mb_status mb_conv_xproj(const void *x, void *state, const float *w, const float *bias, const void *W, void *xc,
+                        void *out, int64_t batch, int64_t width, int32_t n_out, int32_t dtype, void *ws,
+                        size_t ws_bytes, void *stream) {
+    if (batch < 0 || width < 0 || batch > kMaxTokens || width > kMaxTokens) return MB_ERR_INVALID_ARG;
+    if (!mbscan::conv_xproj_supported(width, n_out)) return MB_ERR_UNSUPPORTED;
+    if (batch > kMaxTokens / width) return MB_ERR_INVALID_ARG;
+    if (batch == 0) return MB_OK;
+    if (dtype != MB_BF16) return MB_ERR_UNSUPPORTED;
+    if (!x || !state || !w || !W || !xc || !out || !ws) return MB_ERR_INVALID_ARG;
+    const void *al[] = {x, state, w, bias, W, xc, out};
+    for (const void *q : al)
+        if (q && !aligned16(q)) return MB_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < mb_conv_xproj_workspace_size(batch, width, n_out))
+        return MB_ERR_INVALID_ARG;
+    const int64_t tok = batch * width * 2;
+    const Range rx = range_of(x, tok), rs = range_of(state, 3 * tok), rxc = range_of(xc, tok),
+                ro = range_of(out, batch * n_out * 2), rw = range_of(W, (int64_t)n_out * width * 2),
+                rcw = range_of(w, width * 16), rcb = range_of(bias, width * 4),
+                rws = range_of(ws, (int64_t)mb_conv_xproj_workspace_size(batch, width, n_out));
+    // the written ranges (the first four: xc, out, the window, the scratch) overlap nothing else
+    const Range all[] = {rxc, ro, rs, rws, rx, rw, rcw, rcb};
+    for (int i = 0; i < 4; ++i)
+        for (int j = 0; j < 8; ++j)
+            if (j != i && overlap(all[i], all[j])) return MB_ERR_INVALID_ARG;
+    StatusBlock *sb = static_cast<StatusBlock *>(ws);
+    float *part = reinterpret_cast<float *>(static_cast<char *>(ws) + mbscan::kStatusBytes);
+    return from_cuda(mbscan::launch_conv_xproj(x, state, w, bias, W, xc, out, batch, width, n_out, part, sb,
+                                               (cudaStream_t)stream));
+}
+
 mb_status mb_selftest_timeout(void *ws, size_t ws_bytes, int64_t wait_cycles, void *stream) {
     if (ws == nullptr || ws_bytes < mbscan::kStatusBytes || (reinterpret_cast<uintptr_t>(ws) & 255u))
         return MB_ERR_INVALID_ARG;

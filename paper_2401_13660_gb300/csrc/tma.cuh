@@ -1,5 +1,5 @@
 // Thin wrappers over the sm_90+/sm_100 PTX used for asynchronous staging:
-// mbarriers (with bounded waits) and 3-D TMA tile loads, plus packed f32x2
+// mbarriers (with bounded waits) and 2- to 4-D TMA tile loads and stores, plus packed f32x2
 // arithmetic. Every wait in this library is bounded: a wait that does not
 // complete within kWaitCycles SM clocks returns false and the caller records
 // MB_ERR_TIMEOUT instead of spinning forever.
@@ -115,6 +115,13 @@ __device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, const void 
             reinterpret_cast<uint64_t>(map)),
         "r"(smem_u32(src)), "r"(x), "r"(y), "r"(z)
         : "memory");
+}
+// 2-D tiled TMA store of a shared-memory box (same rules as the 3-D store).
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, const void *src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(smem_u32(src)), "r"(x), "r"(y)
+                 : "memory");
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 // Wait until every committed bulk store has finished reading shared memory.

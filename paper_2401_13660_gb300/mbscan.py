@@ -84,9 +84,14 @@ def load_library(build_if_needed: bool = True) -> ctypes.CDLL:
             lib.mb_scan_backward.argtypes = [ap, vp, vp, vp, ctypes.POINTER(mb_scan_grads), vp, sz, vp]
             lib.mb_selftest_timeout.argtypes = [vp, sz, i64, vp]
             lib.mb_scan_verify_resume.argtypes = [ap, vp, vp, i64, vp, vp, sz, vp]
+            lib.mb_conv_xproj_workspace_size.argtypes = [i64, i64, ctypes.c_int32]
+            lib.mb_conv_xproj_workspace_size.restype = sz
+            lib.mb_conv_xproj.argtypes = [vp, vp, vp, vp, vp, vp, vp, i64, i64, ctypes.c_int32, ctypes.c_int32,
+                                          vp, sz, vp]
             for f in ("mb_scan_prefill", "mb_scan_verify", "mb_rollback", "mb_step", "mb_check",
                       "mb_accept_topk", "mb_step_resume", "mb_scan_prefill_ckpt", "mb_scan_backward",
-                      "mb_rmsnorm", "mb_conv1d_step", "mb_selftest_timeout", "mb_scan_verify_resume"):
+                      "mb_rmsnorm", "mb_conv1d_step", "mb_selftest_timeout", "mb_scan_verify_resume",
+                      "mb_conv_xproj"):
                 getattr(lib, f).restype = ctypes.c_int
             lib.mb_status_string.argtypes = [ctypes.c_int]
             lib.mb_status_string.restype = ctypes.c_char_p
@@ -381,6 +386,34 @@ def mb_conv1d_step(x, state, w, out, *, bias=None, stream=None):
     rc = load_library().mb_conv1d_step(_ptr(x), _ptr(state), _ptr(w), _ptr(bias), _ptr(out), batch, width,
                                        _DTYPES[x.dtype], _stream(stream))
     _check(rc, "mb_conv1d_step")
+    return out
+
+
+def mb_conv_xproj_workspace_size(batch: int, width: int, n_out: int) -> int:
+    """Workspace bytes mb_conv_xproj needs (0: shape not supported)."""
+    return int(load_library().mb_conv_xproj_workspace_size(batch, width, n_out))
+
+
+def mb_conv_xproj(x, state, w, W, xc, out, ws, *, bias=None, stream=None):
+    """Convolution step fused with the x-projection: xc = silu(conv1d_step(x))
+    as mb_conv1d_step (state [batch, 3, width] updated in place), then
+    out = xc W^T. x, xc [batch, width], W [n_out, width], out [batch, n_out],
+    all bf16; w [width, 4], bias [width] fp32; ws a uint8 workspace of
+    mb_conv_xproj_workspace_size bytes."""
+    batch, width = x.shape
+    n_out = W.shape[0]
+    dev, bf = x.device, torch.bfloat16
+    _need(x, "x", bf, (batch, width), dev)
+    _need(state, "state", bf, (batch, 3, width), dev)
+    _need(w, "w", torch.float32, (width, 4), dev)
+    _need(bias, "bias", torch.float32, (width,), dev)
+    _need(W, "W", bf, (n_out, width), dev)
+    _need(xc, "xc", bf, (batch, width), dev)
+    _need(out, "out", bf, (batch, n_out), dev)
+    _need(ws, "ws", torch.uint8, None, dev)
+    rc = load_library().mb_conv_xproj(_ptr(x), _ptr(state), _ptr(w), _ptr(bias), _ptr(W), _ptr(xc), _ptr(out),
+                                      batch, width, n_out, MB_BF16, _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "mb_conv_xproj")
     return out
 
 

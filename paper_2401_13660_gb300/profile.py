@@ -7,7 +7,9 @@ Inputs are drawn on the GPU with the seeded generator of `inputs`; each
 iteration launches the entry point once through the C ABI on one stream.
 Prints the mean device time per launch (CUDA events) and the algorithmic-byte
 rate. For the decode step, `--layers` distinct state/input sets are cycled so
-that the working set exceeds the 129 MB L2 (default 4 layers, 643 MB).
+that the working set exceeds the 129 MB L2 (default 4 layers, 643 MB); the
+fused convolution + x-projection of the decoder (`--entry conv_xproj`) needs
+16 or more of its 8.8 MB window and weight sets for the same (48 in the model).
 """
 from __future__ import annotations
 
@@ -48,17 +50,20 @@ def algorithmic_bytes(entry: str, w, s_in: int) -> int:
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--entry", choices=["prefill", "verify", "rollback", "step", "backward", "decode_model"],
-                    required=True)
+    ap.add_argument("--entry", choices=["prefill", "verify", "rollback", "step", "backward", "decode_model",
+                                        "conv_xproj"], required=True)
     ap.add_argument("--workload", required=True,
-                    help="a workload of inputs.WORKLOADS, or for --entry decode_model a decoder.CONFIGS name")
-    ap.add_argument("--batch", type=int, default=256, help="streams of --entry decode_model")
+                    help="a workload of inputs.WORKLOADS, or for --entry decode_model / conv_xproj a "
+                         "decoder.CONFIGS name")
+    ap.add_argument("--batch", type=int, default=256, help="streams of --entry decode_model / conv_xproj")
     ap.add_argument("--iters", type=int, default=5)
-    ap.add_argument("--layers", type=int, default=4, help="state sets cycled by --entry step")
+    ap.add_argument("--layers", type=int, default=4, help="state sets cycled by --entry step / conv_xproj")
     a = ap.parse_args()
     dev = torch.device("cuda:0")
     if a.entry == "decode_model":
         return decode_model(a, dev)
+    if a.entry == "conv_xproj":
+        return conv_xproj(a, dev)
     w = WORKLOADS[a.workload]
     mb.load_library()
     nsets = a.layers if a.entry == "step" else 1
@@ -155,6 +160,55 @@ def decode_model(a, dev):
     print(json.dumps({"entry": "decode_model", "workload": a.workload, "batch": a.batch, "iters": a.iters,
                       "ms_per_step": round(ms, 4), "bytes_per_step": nb, "GB/s": round(nb / ms / 1e6, 1),
                       "generated_bytes_per_s": round(a.batch / (ms * 1e-3), 1)}))
+
+
+def conv_xproj(a, dev):
+    """The decoder's fused convolution step + x-projection (mb_conv_xproj,
+    with its split-K reduction) at one layer's shapes: one CUDA graph of one
+    launch per each of --layers distinct window and weight sets, replayed
+    --iters times."""
+    from .decoder import CONFIGS
+
+    cfg = CONFIGS[a.workload]
+    B, E, n_out = a.batch, cfg.d_inner, cfg.dt_rank + 2 * cfg.d_state
+    g = torch.Generator(device=dev).manual_seed(3)
+    bf = torch.bfloat16
+    x = torch.randn(B, E, device=dev, generator=g).to(bf)
+    sets = [dict(st=torch.randn(B, 3, E, device=dev, generator=g).to(bf),
+                 w=torch.rand(E, 4, device=dev, generator=g) - 0.5, b=torch.rand(E, device=dev, generator=g) - 0.5,
+                 W=(torch.randn(n_out, E, device=dev, generator=g) / E ** 0.5).to(bf)) for _ in range(a.layers)]
+    xc = torch.empty(B, E, device=dev, dtype=bf)
+    out = torch.empty(B, n_out, device=dev, dtype=bf)
+    ws = torch.zeros(mb.mb_conv_xproj_workspace_size(B, E, n_out), dtype=torch.uint8, device=dev)
+    def run_all():   # one launch per set, as the decoder's layers do
+        for s in sets:
+            mb.mb_conv_xproj(x, s["st"], s["w"], s["W"], xc, out, ws, bias=s["b"])
+
+    stream = torch.cuda.Stream(dev)
+    stream.wait_stream(torch.cuda.current_stream(dev))
+    with torch.cuda.stream(stream):
+        run_all()   # eager warm-up
+    torch.cuda.current_stream(dev).wait_stream(stream)
+    graph = torch.cuda.CUDAGraph()   # replayed, so that host launch costs stay out of the timing
+    with torch.cuda.graph(graph):
+        run_all()
+    graph.replay()
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    ev[0].record()
+    for _ in range(a.iters):
+        graph.replay()
+    ev[1].record()
+    torch.cuda.synchronize()
+    st, _ = mb.mb_check(ws)
+    if st != mb.MB_OK:
+        raise mb.MbError(st, "conv_xproj")
+    us = 1e3 * ev[0].elapsed_time(ev[1]) / max(a.iters * a.layers, 1)
+    # x read, window read and written, xc written, W and the convolution taps read, out written
+    nbytes = B * E * 2 * (1 + 6 + 1) + n_out * E * 2 + E * 20 + B * n_out * 2
+    print(json.dumps({"entry": "conv_xproj", "workload": a.workload, "batch": B, "n_out": n_out, "iters": a.iters,
+                      "us_per_launch": round(us, 3), "algorithmic_bytes": nbytes,
+                      "GB/s": round(nbytes / (us * 1e-6) / 1e9, 1)}))
 
 
 if __name__ == "__main__":

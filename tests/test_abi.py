@@ -342,3 +342,38 @@ def test_noalloc_prefill_host_checks():
     assert _prefill(_args(), h_last=_args().B) == mb.MB_ERR_INVALID_ARG
     # valid arguments: without a GPU the call then fails at its first CUDA call
     assert f(ctypes.byref(_args()), FAKE + (230 << 32), None) in (mb.MB_OK, mb.MB_ERR_CUDA)
+
+
+def test_conv_xproj_host_checks():
+    # mb_conv_xproj: shapes, dtype, alignment, workspace and aliasing are
+    # checked on the host before any CUDA call.
+    lib = mb.load_library()
+    B, W_, n = 256, 4608, 176
+    assert lib.mb_conv_xproj_workspace_size(B, W_, n) == 256 + (W_ // 128) * B * n * 4
+    assert lib.mb_conv_xproj_workspace_size(B, 4600, n) == 0          # width % 128 != 0
+    assert lib.mb_conv_xproj_workspace_size(B, W_, 168) == 0          # no kernel for this n_out
+    need = lib.mb_conv_xproj_workspace_size(B, W_, n)
+    p = {k: FAKE + (i << 32) for i, k in enumerate(("x", "st", "w", "b", "W", "xc", "out", "ws"), start=240)}
+
+    def call(n_out=n, width=W_, batch=B, dtype=mb.MB_BF16, ws_bytes=need, **kw):
+        q = dict(p, **kw)
+        return lib.mb_conv_xproj(q["x"], q["st"], q["w"], q["b"], q["W"], q["xc"], q["out"], batch, width, n_out,
+                                 dtype, q["ws"], ws_bytes, None)
+
+    assert call() in (mb.MB_OK, mb.MB_ERR_CUDA)                     # valid (no GPU here)
+    assert call(b=None) in (mb.MB_OK, mb.MB_ERR_CUDA)               # bias is optional
+    assert call(batch=0) == mb.MB_OK                                # nothing to do
+    assert call(n_out=168) == mb.MB_ERR_UNSUPPORTED
+    assert call(width=4600) == mb.MB_ERR_UNSUPPORTED
+    assert call(dtype=mb.MB_F32) == mb.MB_ERR_UNSUPPORTED
+    assert call(batch=-1) == mb.MB_ERR_INVALID_ARG
+    assert call(ws_bytes=need - 4) == mb.MB_ERR_INVALID_ARG         # workspace too small
+    assert call(ws=p["ws"] + 16) == mb.MB_ERR_INVALID_ARG           # workspace not 256-byte aligned
+    assert call(W=None) == mb.MB_ERR_INVALID_ARG
+    assert call(x=p["x"] + 8) == mb.MB_ERR_INVALID_ARG              # misaligned
+    assert call(xc=p["x"]) == mb.MB_ERR_INVALID_ARG                 # xc is x
+    assert call(out=p["xc"]) == mb.MB_ERR_INVALID_ARG               # out is xc
+    assert call(out=p["st"] + 4096) == mb.MB_ERR_INVALID_ARG        # out inside the window
+    assert call(ws=p["W"]) == mb.MB_ERR_INVALID_ARG                 # workspace over W
+    assert call(st=p["b"] - 256) == mb.MB_ERR_INVALID_ARG           # window runs into the bias
+

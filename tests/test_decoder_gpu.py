@@ -1,4 +1,5 @@
-"""GPU parity of the block kernels (mb_rmsnorm, mb_conv1d_step) and of the
+"""GPU parity of the block kernels (mb_rmsnorm, mb_conv1d_step; mb_conv_xproj
+has its own file) and of the
 whole recurrent decoder (paper_2401_13660_gb300.decoder) against the fp64
 oracle (oracle.rmsnorm, oracle.conv1d_step, oracle.block_step; bf16 casts at
 the tensor boundaries where the GPU path keeps bf16)."""
@@ -129,7 +130,7 @@ def test_decoder_full_size_matches_oracle():
     two bytes, against the fp64 oracle, in three ways:
 
     * each library kernel of every block on the exact tensors the GPU handed
-      it (traced): mb_rmsnorm, mb_conv1d_step, and mb_step whose new SSM state
+      it (traced): mb_rmsnorm, mb_conv_xproj (and the Delta GEMM), and mb_step whose new SSM state
       is held to the fp32-state bar (1e-3) and y to 2e-2;
     * every whole block step (oracle.block_step) on the GPU's inputs to that
       block: block output, convolution window and residual;
@@ -162,7 +163,7 @@ def test_decoder_full_size_matches_oracle():
     ref.check()
     for a, b in zip(dec.ssm + dec.conv, ref.ssm + ref.conv):
         assert torch.equal(a, b)
-    kern = {"rmsnorm": 0.0, "conv_out": 0.0, "step_y": 0.0, "step_state": 0.0}
+    kern = {"rmsnorm": 0.0, "conv_out": 0.0, "xproj": 0.0, "delta": 0.0, "step_y": 0.0, "step_state": 0.0}
     block = {"residual": 0.0, "out": 0.0, "conv": 0.0}
     for l, L in enumerate(dec.layers):
         layer = {k: to_np(L[k]) for k in WEIGHT_KEYS}
@@ -174,6 +175,9 @@ def test_decoder_full_size_matches_oracle():
             xc, cst = oracle.conv1d_step(b["conv"], b["x"], layer["conv_w"], layer["conv_b"])
             assert np.array_equal(b["conv_out"], cst)
             kern["conv_out"] = max(kern["conv_out"], rel_err(tr[l]["xc"], xc))
+            Wx = np.concatenate([layer["W_dtlow"], layer["W_B"], layer["W_C"]])
+            kern["xproj"] = max(kern["xproj"], rel_err(tr[l]["xdbl"], oracle.bf16_round(b["xc"] @ Wx.T)))
+            kern["delta"] = max(kern["delta"], rel_err(tr[l]["dt"], oracle.bf16_round(b["xdbl"][:, :R] @ layer["W_dt"].T)))
             y, st = oracle.step(b["ssm"], x=b["xc"], dt=b["dt"], B=b["xdbl"][:, R:R + N], C=b["xdbl"][:, R + N:],
                                 A=layer["A"], z=b["z"], D=layer["D"], dt_bias=layer["dt_bias"])
             kern["step_y"] = max(kern["step_y"], rel_err(tr[l]["y"], y))
@@ -182,7 +186,7 @@ def test_decoder_full_size_matches_oracle():
             r, out, _, conv = oracle.block_step(layer, b["residual"], b["add"], b["ssm"], b["conv"], eps=cfg.eps)
             for k, want in (("residual", r), ("out", out), ("conv", conv)):
                 block[k] = max(block[k], rel_err(tr[l][k if k == "out" else k + "_out"], want))
-    assert kern["rmsnorm"] <= 1e-2 and kern["conv_out"] <= 1e-2, kern
+    assert max(kern["rmsnorm"], kern["conv_out"], kern["xproj"], kern["delta"]) <= 1e-2, kern
     assert kern["step_y"] <= TOL["bf16"] and kern["step_state"] <= TOL_STATE["bf16"], kern
     assert block["residual"] <= 1e-6 and block["out"] <= 2e-2 and block["conv"] <= 2e-2, block
     want, _, _ = _oracle_decode_layerwise(dec, seq)
