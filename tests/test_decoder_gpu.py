@@ -130,8 +130,9 @@ def test_decoder_full_size_matches_oracle():
     two bytes, against the fp64 oracle, in three ways:
 
     * each library kernel of every block on the exact tensors the GPU handed
-      it (traced): mb_rmsnorm, mb_conv_xproj (and the Delta GEMM), and mb_step whose new SSM state
-      is held to the fp32-state bar (1e-3) and y to 2e-2;
+      it (traced): mb_rmsnorm, mb_conv_xproj (and the Delta GEMM after it),
+      and mb_step whose new SSM state is held to the fp32-state bar (1e-3)
+      and y to 2e-2;
     * every whole block step (oracle.block_step) on the GPU's inputs to that
       block: block output, convolution window and residual;
     * the logits of the whole two-byte decode, end to end.
