@@ -343,8 +343,9 @@ mb_status mb_conv1d_step(const void *x, void *state, const float *w, const float
  *   out    : [batch, n_out] bf16
  *   dtype  : MB_BF16 only (MB_ERR_UNSUPPORTED otherwise)
  *   ws     : 256-byte aligned, ws_bytes >= mb_conv_xproj_workspace_size(
- *            batch, width, n_out): the status block, then the partial sums.
- *            A wait for the W tile that gives up records MB_ERR_TIMEOUT there.
+ *            batch, width, n_out): the status block (zeroed once after
+ *            allocation, as for mb_scan_prefill), then the partial sums. A wait
+ *            for a tile that gives up records MB_ERR_TIMEOUT there.
  * Supported: width % 128 == 0, n_out in {40, 96, 144, 176} (dt_rank + 32
  * for d_state 16 and dt_rank 8, 64, 112, 144); MB_ERR_UNSUPPORTED otherwise.
  * xc, out, state and ws must not overlap one another or the inputs.
