@@ -26,6 +26,11 @@ constexpr int kStepRows = 4;                               // batch rows per til
 #define MB_STEP_STAGES 4
 #endif
 constexpr int kStepStages = MB_STEP_STAGES;
+// Tiles per CTA whose state is prefetched into L2 before the dependency wait
+// (measured at batch 256 x 4608: 1 / 2 / 4 tiles took the back-to-back step
+// from 27.6 to 26.4 / 25.8 / 25.8 us and the whole-model decode, where a GEMM
+// precedes each step, from 2.885 to 2.849 / 2.834 / 2.926 ms).
+constexpr int kStepPrefetch = 2;
 
 // One tile of the decode step in shared memory (TMA destinations; every member
 // offset is a multiple of 128 bytes for both dtypes).
@@ -102,7 +107,9 @@ __device__ __forceinline__ float4 lds4(const __nv_bfloat16 *p) {
 // the 4-lane reduction owns row q's output. New states go straight from
 // registers to global memory (512 contiguous bytes per warp and row). The
 // round-robin order changes the channel block from tile to tile, so each
-// lane loads its channel's A row, dt_bias and D one tile ahead.
+// lane loads its channel's A row, dt_bias and D one tile ahead. Launched with
+// programmatic dependent launch, the producer prefetches its first tiles'
+// state into L2 while the previous kernel drains.
 // kResume (speculative decoding, after the bifurcation of Algorithm 1): row s
 // starts from h0[s] or h_all[s, accept[s]-1] instead of the state itself, so
 // the rollback needs no copy of its own; rows with an accept count outside
@@ -125,6 +132,18 @@ __global__ void __launch_bounds__(kStepThreads, sizeof(T) == 2 ? 3 : 2) step_ker
     }
     __syncthreads();
     pdl_trigger();   // persistent grid: the next kernel's CTAs take the SMs as this one drains
+    // The state of this CTA's first kStepPrefetch tiles is prefetched into L2
+    // before the wait for the previous kernel: the first loads after the wait
+    // then come from L2 instead of paying the DRAM latency while the previous
+    // kernel drains. A prefetch returns nothing, so whatever that kernel still
+    // writes is seen by the loads after the wait.
+    if (!kResume && warp == kStepConsumers && lane == 0) {
+        for (int j = 0; j < kStepPrefetch; ++j) {
+            const int k = blockIdx.x + j * gridDim.x;
+            if (k >= a.ntiles) break;
+            tma_prefetch_3d(&a.tm_state, 0, (k % a.ntiles_d) * kStepCh, (k / a.ntiles_d) * kStepRows);
+        }
+    }
     pdl_wait();      // everything below reads or writes global memory
 
     if (warp == kStepConsumers) {
