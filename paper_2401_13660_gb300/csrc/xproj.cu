@@ -11,7 +11,9 @@
 // split over K: CTA (m, s) owns batch rows 64 m .. 64 m + 63 and channels
 // 128 s .. 128 s + 127. One thread issues all of its global traffic as TMA
 // copies at the start: the x tile, the three window tiles and the matching
-// 128 columns of W (two 64-column boxes, 128-byte swizzle). As soon as x and
+// 128 columns of W (two 64-column boxes, 128-byte swizzle); the window and W
+// tiles, which the preceding input GEMM does not produce, are first prefetched
+// into L2 while that kernel drains (programmatic dependent launch). As soon as x and
 // the window have landed, the shifted window goes back out as three TMA
 // stores of the tiles just loaded (s1, s2, x), while the threads compute the
 // convolution step from shared memory into the A operand (bf16, the same
@@ -79,6 +81,12 @@ __global__ void __launch_bounds__(kXpThreads) conv_xproj_kernel(const __grid_con
         fence_mbar_init();
     }
     __syncthreads();
+    if (tid == 0) {   // the window and W tiles into L2 while the previous kernel (the input GEMM) drains
+#pragma unroll
+        for (int j = 0; j < 3; ++j) tma_prefetch_3d(&a.tm_s, k0, j, r0);
+        tma_prefetch_2d(&a.tm_w, k0, 0);
+        tma_prefetch_2d(&a.tm_w, k0 + 64, 0);
+    }
     pdl_wait();   // everything below reads or writes global memory
     if (tid == 0) {
         mbar_arrive_expect_tx(&bar[0], 4 * kXpTile);
