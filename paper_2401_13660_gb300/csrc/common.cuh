@@ -78,9 +78,10 @@ __device__ __forceinline__ float2 ldg2(const __nv_bfloat16 *p) {
 
 // ---- Programmatic dependent launch. Kernels launched with launch_pdl may
 // start while the previous kernel on the stream is still draining; each such
-// kernel runs pdl_wait() before its first global-memory access, which returns
-// once every prerequisite grid has completed and its writes are visible, so
-// only shared-memory set-up overlaps the predecessor. pdl_trigger() lets the
+// kernel runs pdl_wait() before its first global-memory read or write, which
+// returns once every prerequisite grid has completed and its writes are
+// visible, so only shared-memory set-up and L2 prefetches (hints that return
+// no data) overlap the predecessor. pdl_trigger() lets the
 // next kernel launch before this one completes (it still waits for it). Only
 // the persistent decode step and the single-wave fused convolution +
 // x-projection issue it: a grid of many short-lived CTAs that triggers early
