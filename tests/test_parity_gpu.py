@@ -285,3 +285,51 @@ def test_step_rows_independent_of_the_launch_shape():
     small = {k: (v[:4].contiguous() if torch.is_tensor(v) and v.shape[0] == 256 else v) for k, v in inp.items()}
     ry, rh, _ = oracle_scan(small)
     assert rel_err(outs[4][0], ry) <= TOL["bf16"] and rel_err(outs[4][1], rh) <= TOL_STATE["bf16"]
+
+
+@pytest.mark.parametrize("rows", [256, 32, 4])
+def test_back_to_back_steps_on_one_state(rows):
+    """Consecutive mb_step launches on the same state with nothing in between:
+    each step kernel may start (and prefetch its first tiles' state into L2)
+    while the previous one still writes that state. 16 steps launched back to
+    back, eagerly and from a CUDA graph, must equal bit for bit the same steps
+    with a device synchronisation after each, and the oracle's 16-step scan.
+    256 rows x 2048 channels fill the resident CTA slots; 32 and 4 rows leave
+    slots free, so consecutive grids can be resident together."""
+    L = 16
+    inp = make_inputs(rows, L, 2048, 16, "bf16", "normal", seed=54 + rows, device=DEV)
+    sl = lambda k, t: inp[k][:, t:t + 1].contiguous()
+    steps = [dict(x=sl("x", t), dt=sl("dt", t), B=sl("B", t), C=sl("C", t), z=sl("z", t)) for t in range(L)]
+    ys = [torch.empty_like(s["x"]) for s in steps]
+
+    def run(state, sync):
+        for s, y in zip(steps, ys):
+            mb.mb_step(s["x"], s["dt"], s["B"], s["C"], inp["A"], y, state, z=s["z"], D=inp["D"],
+                       dt_bias=inp["dt_bias"])
+            if sync:
+                torch.cuda.synchronize()
+        return torch.cat(ys, 1).clone()
+
+    st_sync = inp["h0"].clone()
+    y_sync = run(st_sync, True)
+    st_eager = inp["h0"].clone()
+    y_eager = run(st_eager, False)
+    torch.cuda.synchronize()
+    st_graph = inp["h0"].clone()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        run(inp["h0"].clone(), False)   # warm-up outside the capture
+    torch.cuda.current_stream().wait_stream(side)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for s, y in zip(steps, ys):
+            mb.mb_step(s["x"], s["dt"], s["B"], s["C"], inp["A"], y, st_graph, z=s["z"], D=inp["D"],
+                       dt_bias=inp["dt_bias"])
+    g.replay()
+    torch.cuda.synchronize()
+    y_graph = torch.cat(ys, 1).clone()
+    assert torch.equal(y_eager, y_sync) and torch.equal(st_eager, st_sync)
+    assert torch.equal(y_graph, y_sync) and torch.equal(st_graph, st_sync)
+    ry, rh, _ = oracle_scan(inp)
+    assert rel_err(y_sync, ry) <= TOL["bf16"] and rel_err(st_sync, rh) <= TOL_STATE["bf16"]
