@@ -102,3 +102,53 @@ def test_conv_xproj_in_place_of_the_unfused_pair():
     assert torch.equal(xa, xb) and torch.equal(sa, sb)
     assert rel_err(oa, to_np(ob)) <= 2.0 ** -7
 
+
+
+@pytest.mark.parametrize("batch", [256, 4])
+def test_back_to_back_calls_on_one_window(batch):
+    """Consecutive mb_conv_xproj calls on the same convolution window with
+    nothing in between (each call may start, and prefetch its window tiles
+    into L2, while the previous one still writes them): eagerly and from a CUDA
+    graph they equal bit for bit the same calls with a device synchronisation
+    after each, and the window ends as the oracle's."""
+    width, n_out, T = 4608, 176, 6
+    g, w, bias, W = _weights(width, n_out, 21 + batch)
+    xs = [torch.randn(batch, width, device=DEV, generator=g).to(BF) for _ in range(T)]
+    s0 = torch.randn(batch, 3, width, device=DEV, generator=g).to(BF)
+    xcs = [torch.empty_like(x) for x in xs]
+    outs = [torch.empty(batch, n_out, device=DEV, dtype=BF) for _ in range(T)]
+    ws = torch.zeros(mb.mb_conv_xproj_workspace_size(batch, width, n_out), dtype=torch.uint8, device=DEV)
+
+    def run(state, sync):
+        for x, xc, out in zip(xs, xcs, outs):
+            mb.mb_conv_xproj(x, state, w, W, xc, out, ws, bias=bias)
+            if sync:
+                torch.cuda.synchronize()
+        return [t.clone() for t in xcs + outs]
+
+    st_sync = s0.clone()
+    r_sync = run(st_sync, True)
+    st_eager = s0.clone()
+    r_eager = run(st_eager, False)
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        run(s0.clone(), False)   # warm-up outside the capture
+    torch.cuda.current_stream().wait_stream(side)
+    st_graph = s0.clone()
+    gr = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gr):
+        for x, xc, out in zip(xs, xcs, outs):
+            mb.mb_conv_xproj(x, st_graph, w, W, xc, out, ws, bias=bias)
+    gr.replay()
+    torch.cuda.synchronize()
+    r_graph = [t.clone() for t in xcs + outs]
+    for a, b in zip(r_eager + r_graph, r_sync + r_sync):
+        assert torch.equal(a, b)
+    assert torch.equal(st_eager, st_sync) and torch.equal(st_graph, st_sync)
+    st_np = to_np(s0)
+    for x in xs:
+        _, st_np = oracle.conv1d_step(st_np, to_np(x), to_np(w), to_np(bias))
+    assert np.array_equal(to_np(st_sync), st_np)
+    assert mb.mb_check(ws) == (mb.MB_OK, -1)
